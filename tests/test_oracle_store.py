@@ -1,0 +1,339 @@
+"""Pins of the oracle store (CPU only).
+
+The store's results are fixed by identities and invariants the paper's
+statement of the problem gives (written once, read back unchanged, reclaimed
+when freed; §5.2, §5.3) and by the readings of its silent points listed in
+the oracle's header. Each check here is computed independently of the
+oracle's own bookkeeping:
+
+* get(put(x)) == x, with the bytes read back from an explicit pool array
+  through the page lists (brute force) and compared with the input;
+* no two live objects share a page, every page is below the capacity, and the
+  free stack is exactly the complement of the used pages;
+* pages in use == sum of ceil(n / P), with ceil counted by a loop;
+* compaction keeps every object's bytes, leaves every page below the limit,
+  moves exactly the live pages at or above the limit, into the lowest free
+  pages, and copies exactly the valid bytes;
+* hand-derived traces for placement (LIFO) and for LRU victims in reverse
+  layer order (§5.3, "How does it work?").
+
+Planted mistakes in the oracle must fail these checks.
+"""
+import itertools
+
+import numpy as np
+import pytest
+
+import oracle.store as ostore
+from oracle import EVICTED, INVALID, NOSPACE, NOT_FOUND, OK, OracleStore, PutItem
+
+
+def ceil_pages_by_counting(n, P):
+    k = 0
+    while k * P < n:
+        k += 1
+    return k
+
+
+def check_invariants(s: OracleStore, inputs: dict):
+    """inputs: id -> the bytes that were put (None for reserved objects)."""
+    P = s.page_bytes
+    seen = {}
+    for oid, o in s.objects.items():
+        assert len(o.pages) == ceil_pages_by_counting(o.nbytes, P)
+        for p in o.pages:
+            assert 0 <= p < s.limit_pages, "page outside the capacity"
+            assert p not in seen, f"page {p} shared by {seen.get(p)} and {oid}"
+            seen[p] = oid
+    used = sum(ceil_pages_by_counting(o.nbytes, P) for o in s.objects.values())
+    assert s.used_pages() == used
+    assert len(s.free_stack) == len(set(s.free_stack))
+    assert set(s.free_stack) | set(seen) == set(range(s.limit_pages))
+    assert not (set(s.free_stack) & set(seen))
+    assert set(s.objects) == set(inputs)
+    # brute force read through the page lists of the explicit pool
+    if s.pool is not None:
+        for oid, want in inputs.items():
+            if want is None:
+                continue
+            o = s.objects[oid]
+            got = np.concatenate([s.pool[p * P:p * P + min(P, o.nbytes - j * P)] for j, p in enumerate(o.pages)]) \
+                if o.pages else np.zeros(0, np.uint8)
+            assert np.array_equal(got, want)
+
+
+def random_ops(seed, P, total_pages, n_ops, max_pages=3, check=True):
+    g = np.random.default_rng(seed)
+    s = OracleStore(total_pages * P, P, paged_pool=True)
+    inputs = {}
+    for _ in range(n_ops):
+        r = g.random()
+        if r < 0.45:
+            k = int(g.integers(1, 4))
+            items = []
+            for _ in range(k):
+                n = int(g.integers(0, max_pages * P + 1))
+                data = None if g.random() < 0.1 else g.integers(0, 256, n, dtype=np.uint8)
+                items.append(PutItem(n, data, group=int(g.integers(0, 3)), order=int(g.integers(0, 4)),
+                                     evictable=bool(g.random() < 0.5)))
+            free_before = s.free_pages()
+            evictable_pages = sum(ceil_pages_by_counting(o.nbytes, P) for o in s.objects.values()
+                                  if o.evictable and o.group not in {it.group for it in items})
+            demand = sum(ceil_pages_by_counting(it.nbytes, P) for it in items)
+            snap = (dict((k2, list(v.pages)) for k2, v in s.objects.items()), list(s.free_stack), s.next_id)
+            st, ids = s.put_batch(items)
+            if demand > free_before + evictable_pages:
+                assert st == NOSPACE
+                assert snap == (dict((k2, list(v.pages)) for k2, v in s.objects.items()), list(s.free_stack),
+                                s.next_id), "a failed put changed the store"
+            else:
+                assert st == OK
+                for v in s.last_evictions:
+                    inputs.pop(v)
+                for oid, it in zip(ids, items):
+                    inputs[oid] = None if it.data is None else it.data.copy()
+        elif r < 0.7 and inputs:
+            ids = list(g.choice(list(inputs), size=min(len(inputs), int(g.integers(1, 4))), replace=False))
+            st, per, outs = s.get_batch(ids)
+            assert st == OK
+            for oid, out in zip(ids, outs):
+                if inputs[int(oid)] is not None:
+                    assert np.array_equal(out, inputs[int(oid)])
+        elif r < 0.9 and inputs:
+            ids = list(g.choice(list(inputs), size=min(len(inputs), int(g.integers(1, 3))), replace=False))
+            assert s.free(ids) == OK
+            for oid in ids:
+                inputs.pop(int(oid))
+        else:
+            limit = int(g.integers(0, total_pages + 1))
+            own_before = {p: (oid, j) for oid, o in s.objects.items() for j, p in enumerate(o.pages)}
+            used = len(own_before)
+            st, moves = s.compact(limit * P)
+            if used > limit:
+                assert st == NOSPACE and moves == []
+            else:
+                assert st == OK
+                tail = sorted(p for p in own_before if p >= limit)
+                assert [m[0] for m in moves] == tail
+                free_head = [p for p in range(limit) if p not in own_before]
+                assert [m[1] for m in moves] == free_head[:len(tail)]
+                for src, dst, valid in moves:
+                    oid, j = own_before[src]
+                    n = s.objects[oid].nbytes
+                    assert valid == min(P, n - j * P)
+                    assert s.objects[oid].pages[j] == dst
+                # the free stack pops the lowest page first
+                assert s.free_stack == sorted(s.free_stack, reverse=True)
+        if check:
+            check_invariants(s, inputs)
+    return s, inputs
+
+
+@pytest.mark.parametrize("seed", range(12))
+@pytest.mark.parametrize("P", [64, 256, 4096])
+def test_random_sequences_tiny_pools(seed, P):
+    random_ops(seed, P, total_pages=8 + seed * 4, n_ops=120)
+
+
+def test_exhaustive_two_op_sequences():
+    """Every pair of (put size, free/compact choice) on a 4-page pool of 64 B
+    pages: brute force over a small op alphabet."""
+    P = 64
+    sizes = [0, 1, 63, 64, 65, 128, 191, 256]
+    for a, b, c in itertools.product(sizes, sizes, range(5)):
+        s = OracleStore(4 * P, P, paged_pool=True)
+        inputs = {}
+        for n in (a, b):
+            data = np.arange(n, dtype=np.uint8) ^ (n & 0xFF)
+            st, ids = s.put_batch([PutItem(n, data)])
+            if st == OK:
+                inputs[ids[0]] = data
+            else:
+                assert st == NOSPACE
+                assert sum(ceil_pages_by_counting(len(v), P) for v in inputs.values()) + \
+                    ceil_pages_by_counting(n, P) > 4
+        check_invariants(s, inputs)
+        if inputs:
+            first = min(inputs)
+            assert s.free([first]) == OK
+            inputs.pop(first)
+        st, _ = s.compact(c * P)
+        assert st == (OK if s.used_pages() <= c else NOSPACE)
+        check_invariants(s, inputs)
+
+
+def test_lifo_placement_hand_trace():
+    """Pages worked out by hand from readings 2 and 7 (1 KiB pages, 8 pages)."""
+    P = 1024
+    s = OracleStore(8 * P, P, paged_pool=True)
+    _, (a,) = s.put_batch([PutItem(2500, np.full(2500, 1, np.uint8))])
+    assert s.pages_of(a) == [0, 1, 2]
+    _, (b,) = s.put_batch([PutItem(1024, np.full(1024, 2, np.uint8))])
+    assert s.pages_of(b) == [3]
+    assert s.free([a]) == OK
+    assert s.free_stack == [7, 6, 5, 4, 0, 1, 2]
+    _, (c,) = s.put_batch([PutItem(2048, np.full(2048, 3, np.uint8))])
+    assert s.pages_of(c) == [2, 1]
+    d_bytes = np.arange(3000, dtype=np.uint8)
+    _, (d,) = s.put_batch([PutItem(3000, d_bytes)])
+    assert s.pages_of(d) == [0, 4, 5]
+    assert s.compact(4 * P) == (NOSPACE, [])
+    assert s.free([b]) == OK
+    st, moves = s.compact(5 * P)
+    assert st == OK and moves == [(5, 3, 3000 - 2048)]
+    assert s.pages_of(d) == [0, 4, 3] and s.free_stack == []
+    assert s.put_batch([PutItem(1, np.zeros(1, np.uint8))])[0] == NOSPACE
+    st, moves = s.compact(8 * P)
+    assert st == OK and moves == [] and s.free_stack == [7, 6, 5]
+    _, (e,) = s.put_batch([PutItem(1, np.zeros(1, np.uint8))])
+    assert s.pages_of(e) == [5]
+    _, _, (out,) = s.get_batch([d])
+    assert np.array_equal(out, d_bytes)
+    assert s.stats["pages_moved"] == 1 and s.stats["bytes_moved"] == 952
+
+
+def test_lru_reverse_layer_hand_trace():
+    """Victims worked out by hand from §5.3 (LRU model first, last layers
+    first) and reading 6 (1 KiB pages, 6 pages)."""
+    P = 1024
+    s = OracleStore(6 * P, P)
+    st, w1 = s.put_batch([PutItem(P, np.zeros(P, np.uint8), group=1, order=k, evictable=True) for k in range(3)])
+    assert st == OK and w1 == [1, 2, 3]
+    st, w2 = s.put_batch([PutItem(P, np.zeros(P, np.uint8), group=2, order=k, evictable=True) for k in range(2)])
+    assert w2 == [4, 5] and [s.pages_of(i)[0] for i in w1 + w2] == [0, 1, 2, 3, 4]
+    assert s.get_batch([1])[0] == OK            # model 1 is now the most recent
+    st, (x,) = s.put_batch([PutItem(3 * P, np.zeros(3 * P, np.uint8), group=3)])
+    assert st == OK and s.last_evictions == [5, 4]   # model 2 first, layer 1 before layer 0
+    assert s.pages_of(x) == [3, 4, 5]
+    st, per, _ = s.get_batch([4, 99, 1])
+    assert st == EVICTED and per == [EVICTED, NOT_FOUND, OK]
+    st, (y,) = s.put_batch([PutItem(P, np.zeros(P, np.uint8), group=2, order=0, evictable=True)])
+    assert st == OK and s.last_evictions == [3]      # group 2 is pinned by this put; layer 2 of model 1
+    assert s.pages_of(y) == [2]
+    before = sorted(s.objects)
+    st, _ = s.put_batch([PutItem(4 * P, np.zeros(4 * P, np.uint8), group=4)])
+    assert st == NOSPACE and s.last_evictions == [] and sorted(s.objects) == before
+    # ties inside a group go to the highest id
+    s2 = OracleStore(2 * P, P)
+    s2.put_batch([PutItem(P, np.zeros(P, np.uint8), group=5, order=1, evictable=True) for _ in range(2)])
+    st, _ = s2.put_batch([PutItem(P, np.zeros(P, np.uint8), group=6)])
+    assert st == OK and s2.last_evictions == [2]
+    # freeing an evicted id drops it; its get is then NOT_FOUND
+    assert s.free([4]) == OK and s.get_batch([4])[0] == NOT_FOUND
+
+
+def test_error_paths_change_nothing():
+    P = 256
+    s = OracleStore(4 * P, P)
+    st, ids = s.put_batch([PutItem(10, np.zeros(10, np.uint8)), PutItem(300, np.zeros(300, np.uint8))])
+    assert st == OK and ids == [1, 2]
+    assert s.put_batch([PutItem(5, np.zeros(4, np.uint8))])[0] == INVALID
+    assert s.free([1, 1]) == INVALID and 1 in s.objects
+    assert s.free([1, 77]) == NOT_FOUND and 1 in s.objects
+    assert s.get_batch([2], casts=[1])[0] == OK          # 300 % 4 == 0
+    assert s.get_batch([1], casts=[1])[0] == INVALID     # 10 % 4 != 0
+    assert s.get_batch([1], casts=[2])[0] == INVALID
+    assert s.compact(100)[0] == INVALID                  # not a page multiple
+    assert s.compact(5 * P)[0] == INVALID                # beyond the pool
+    st, per, outs = s.get_batch([1, 1, 2])               # repeats are allowed
+    assert st == OK and len(outs) == 3
+    assert s.next_id == 3
+
+
+def test_zero_byte_and_reserved_objects():
+    s = OracleStore(4 * 64, 64, paged_pool=True)
+    st, (z, r) = s.put_batch([PutItem(0, np.zeros(0, np.uint8)), PutItem(100, None)])
+    assert st == OK and s.pages_of(z) == [] and len(s.pages_of(r)) == 2
+    st, _, outs = s.get_batch([z])
+    assert st == OK and outs[0].size == 0
+    check_invariants(s, {z: np.zeros(0, np.uint8), r: None})
+
+
+def test_cast_on_get_matches_cast_module():
+    s = OracleStore(1 << 20, 4096)
+    x = np.random.default_rng(0).standard_normal(3000).astype(np.float32)
+    _, (i,) = s.put_batch([PutItem(x.nbytes, x.view(np.uint8))])
+    _, _, (out,) = s.get_batch([i], casts=[1])
+    import torch
+    assert np.array_equal(out.view(np.uint16), torch.from_numpy(x).to(torch.bfloat16).view(torch.int16).numpy().view(np.uint16))
+
+
+# -- planted mistakes -------------------------------------------------------------
+
+def _expect_failure(fn):
+    try:
+        fn()
+    except AssertionError:
+        return True
+    return False
+
+
+def test_planted_floor_pages(monkeypatch):
+    monkeypatch.setattr(ostore, "pages_for", lambda n, P: int(n) // int(P))
+    assert _expect_failure(lambda: random_ops(1, 64, 12, 60))
+
+
+def test_planted_reversed_free_push(monkeypatch):
+    def release(self, oid):
+        for p in reversed(self.objects[oid].pages):
+            self.free_stack.append(p)
+        del self.objects[oid]
+    monkeypatch.setattr(OracleStore, "_release", release)
+    assert _expect_failure(test_lifo_placement_hand_trace)
+
+
+def test_planted_victims_lowest_layer_first(monkeypatch):
+    orig = OracleStore._victims
+
+    def victims(self, demand, pinned):
+        v = orig(self, demand, pinned)
+        if not v:
+            return v
+        cands = sorted((o for o in self.objects if self.objects[o].evictable and self.objects[o].group not in pinned),
+                       key=lambda o: (self.group_last[self.objects[o].group], self.objects[o].order, o))
+        return cands[:len(v)]
+    monkeypatch.setattr(OracleStore, "_victims", victims)
+    assert _expect_failure(test_lru_reverse_layer_hand_trace)
+
+
+def test_planted_compaction_to_highest_free(monkeypatch):
+    orig = OracleStore.compact
+
+    def compact(self, limit_bytes):
+        # moves to the highest free pages instead of the lowest
+        limit = int(limit_bytes) // self.page_bytes
+        if int(limit_bytes) % self.page_bytes or limit > self.total_pages or self.used_pages() > limit:
+            return orig(self, limit_bytes)
+        own = self.owners()
+        tail = sorted(p for p in own if p >= limit)
+        head = [p for p in range(limit - 1, -1, -1) if p not in own]
+        moves = []
+        for src, dst in zip(tail, head):
+            oid, j = own[src]
+            o = self.objects[oid]
+            valid = min(self.page_bytes, o.nbytes - j * self.page_bytes)
+            o.pages[j] = dst
+            if self.pool is not None:
+                P = self.page_bytes
+                self.pool[dst * P:dst * P + valid] = self.pool[src * P:src * P + valid]
+            moves.append((src, dst, valid))
+        own = self.owners()
+        self.free_stack = [p for p in range(limit - 1, -1, -1) if p not in own]
+        self.limit_pages = limit
+        return OK, moves
+    monkeypatch.setattr(OracleStore, "compact", compact)
+    assert _expect_failure(test_lifo_placement_hand_trace)
+    assert _expect_failure(lambda: [random_ops(sd, 64, 16, 150) for sd in range(6)])
+
+
+def test_planted_compaction_drops_bytes(monkeypatch):
+    orig = OracleStore.compact
+
+    def compact(self, limit_bytes):
+        st, moves = orig(self, limit_bytes)
+        if self.pool is not None:
+            for src, dst, valid in moves:   # forget the last byte of each moved page
+                self.pool[dst * self.page_bytes + valid - 1] ^= 0xFF
+        return st, moves
+    monkeypatch.setattr(OracleStore, "compact", compact)
+    assert _expect_failure(lambda: [random_ops(sd, 64, 16, 150) for sd in range(6)])
