@@ -1,0 +1,444 @@
+"""Benchmark of the paged tensor store on GB300.
+
+Workload (default): the T2I intermediate handoff -- 8 GiB pool of 2 MiB pages,
+64 requests in flight, each handing on bf16 text embeddings [B,512,4096],
+bf16 pooled embeddings [B,768], fp32 latents [B,16,128,128] (got with the
+fused fp32 -> bf16 RNE cast) and fp16 decoded images [B,3,1024,1024]; B = 8.
+One step = put all 64 requests from producer buffers, get all 64 into consumer
+buffers, free everything: 128 batched calls, each one kernel launch.
+
+Metric: algorithmic read + write bytes / time (put and get: 2 x payload,
+cast get: 1.5 x the fp32 payload), GB/s, and its fraction of the measured
+HBM copy rate. The inputs of one step (5.5 GiB read, 5.5 GiB written) are
+far larger than L2, so no L2 flush is needed between steps.
+
+  python bench.py [--gpus N --steps K --warmup W] [--impl reference]
+
+Under torchrun each rank runs an independent store on its own GPU (the store
+has no cross-GPU step); rank 0 prints one JSON line with the whole-job value.
+"""
+from __future__ import annotations
+
+import argparse
+import ctypes as C
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+import workloads as W  # noqa: E402
+
+METRIC = "batched get/put/compact GB/s (read+write bytes) and % of GB300 HBM peak"
+FALLBACK_HBM_GBS = 6800.0
+
+
+def parse():
+    p = argparse.ArgumentParser()
+    p.add_argument("--gpus", type=int, default=1)
+    p.add_argument("--steps", type=int, default=10)
+    p.add_argument("--warmup", type=int, default=3)
+    p.add_argument("--impl", default="native", choices=["native", "reference"])
+    p.add_argument("--batch", type=int, default=8, help="B of the handoff workload")
+    p.add_argument("--requests", type=int, default=64)
+    p.add_argument("--no-e2e", action="store_true")
+    p.add_argument("--no-cpu", action="store_true")
+    p.add_argument("--sweep", action="store_true", help="also time B = 1 and B = 4")
+    return p.parse_args()
+
+
+# ----------------------------------------------------------------------------- helpers
+def peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(path):
+        with open(path) as f:
+            d = json.load(f)
+        return float(d["hbm_gbs"]), "measured"
+    return FALLBACK_HBM_GBS, "fallback"
+
+
+def ncu_traffic(kernel: str, launch: str):
+    """dram read+write bytes of one ``kernel`` launch of shape ``launch`` from
+    the committed ncu summary, if it was taken on the current kernel source
+    (else None)."""
+    from paper_2607_26566_gb300 import build as b
+
+    path = os.path.join(ROOT, "profiles", "traffic.txt")
+    if not os.path.exists(path):
+        return None
+    src_hash = b.kernel_source_hash()
+    for line in open(path):
+        f = dict(kv.split("=", 1) for kv in line.split() if "=" in kv)
+        if f.get("kernel") == kernel and f.get("launch") == launch and f.get("source") == src_hash:
+            return float(f["dram_bytes_per_launch"])
+    return None
+
+
+class Clocks:
+    """nvidia-smi sampling of SM clocks and throttle reasons during a region."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index: int):
+        self.index = index
+        self.proc = None
+        self.lines = []
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(["nvidia-smi", "-i", str(self.index), "--query-gpu=" + self.FIELDS,
+                                          "--format=csv,noheader,nounits", "-lms", "100"],
+                                         stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.t = threading.Thread(target=self._read, daemon=True)
+            self.t.start()
+        except OSError:
+            self.proc = None
+        return self
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def __exit__(self, *a):
+        if self.proc:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+
+    def summary(self):
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in self.lines:
+            f = [x.strip() for x in line.split(",")]
+            if len(f) < 9:
+                continue
+            try:
+                sm.append(float(f[1]))
+                mx.append(float(f[2]))
+            except ValueError:
+                continue
+            for n, v in zip(names, f[5:9]):
+                if v.lower().startswith("active"):
+                    reasons.add(n)
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": [], "samples": 0}
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx), "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+# ----------------------------------------------------------------------------- handoff
+class Handoff:
+    """The handoff workload bound to one store. Descriptor arrays are built
+    once; a step issues raw C-ABI calls only."""
+
+    def __init__(self, B: int, requests: int, device, host_buffers: bool = False, seed: int = 0):
+        import torch
+
+        from paper_2607_26566_gb300 import Store, get_descs, put_descs
+
+        C_ = W.HANDOFF
+        self.torch = torch
+        self.device = device
+        self.specs = W.handoff_specs(B)
+        self.n_obj = len(self.specs)
+        self.requests = requests
+        self.ci = W.handoff_cast_index()
+        self.pool = torch.empty(C_["pool_bytes"], dtype=torch.uint8, device=device)
+        self.store = Store(self.pool, C_["page_bytes"])
+        self.lib = self.store._lib
+        self.h = self.store._h
+        self.inputs, self.outputs = [], []
+        for r in range(requests):
+            ts = W.handoff_request_torch(seed, r, self.specs, device)
+            outs = [torch.empty(sp.nbytes // (2 if j == self.ci else 1), dtype=torch.uint8, device=device)
+                    for j, sp in enumerate(self.specs)]
+            if host_buffers:
+                ts = [t.cpu().pin_memory() for t in ts]
+                outs = [torch.empty(o.numel(), dtype=torch.uint8).pin_memory() for o in outs]
+            self.inputs.append(ts)
+            self.outputs.append(outs)
+        torch.cuda.synchronize(device)
+        self.ids = np.zeros(requests * self.n_obj, np.uint64)
+        self.pd = [put_descs(ts, nbytes=[sp.nbytes for sp in self.specs], src_is_host=int(host_buffers),
+                             dtype_tag=[sp.dtype_tag for sp in self.specs]) for ts in self.inputs]
+        casts = [1 if j == self.ci else 0 for j in range(self.n_obj)]
+        self.gd = [get_descs(np.zeros(self.n_obj, np.uint64), outs, cast=casts) for outs in self.outputs]
+        self.pd_p = [d.ctypes.data for d in self.pd]
+        self.gd_p = [d.ctypes.data for d in self.gd]
+        self.ids_p = [self.ids.ctypes.data + 8 * self.n_obj * r for r in range(requests)]
+        payload = sum(sp.nbytes for sp in self.specs)
+        lat = self.specs[self.ci].nbytes
+        self.put_bytes = 2 * payload * requests
+        self.get_bytes = (2 * (payload - lat) + 1.5 * lat) * requests
+        self.h2d_bytes = payload * requests
+        self.d2h_bytes = (payload - lat // 2) * requests
+        self.step_bytes = self.put_bytes + self.get_bytes
+
+    def step(self, stream, ev=None):
+        lib, h, n = self.lib, self.h, self.n_obj
+        s = C.c_void_p(stream)
+        for r in range(self.requests):
+            if ev is not None:
+                ev["put"][r][0].record()
+            st = lib.t2i_put_batch(h, C.c_void_p(self.pd_p[r]), n, C.c_void_p(self.ids_p[r]), s)
+            if ev is not None:
+                ev["put"][r][1].record()
+            if st:
+                raise RuntimeError("put_batch: " + self.store.last_error())
+        for r in range(self.requests):
+            self.gd[r]["id"] = self.ids[n * r:n * (r + 1)]
+            if ev is not None:
+                ev["get"][r][0].record()
+            st = lib.t2i_get_batch(h, C.c_void_p(self.gd_p[r]), n, None, s)
+            if ev is not None:
+                ev["get"][r][1].record()
+            if st:
+                raise RuntimeError("get_batch: " + self.store.last_error())
+        st = lib.t2i_free(h, C.c_void_p(self.ids.ctypes.data), len(self.ids))
+        if st:
+            raise RuntimeError("free: " + self.store.last_error())
+
+    def verify(self):
+        """get(put(x)) == x on every non-cast output after a step (cheap)."""
+        torch = self.torch
+        for ts, outs in zip(self.inputs, self.outputs):
+            for j, (t, o) in enumerate(zip(ts, outs)):
+                if j != self.ci and not torch.equal(t.reshape(-1).view(torch.uint8), o.reshape(-1)):
+                    raise RuntimeError("handoff output differs from its input")
+
+
+def time_handoff(hw: Handoff, steps: int, warmup: int, dist_ctx, per_kernel: bool, clocks_index=None):
+    torch = hw.torch
+    stream = torch.cuda.current_stream(hw.device)
+    for _ in range(warmup):
+        hw.step(stream.cuda_stream)
+    torch.cuda.synchronize(hw.device)
+    ev = None
+    if per_kernel:
+        mk = lambda: [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+                      for _ in range(hw.requests)]
+        evs = [{"put": mk(), "get": mk()} for _ in range(steps)]
+    launches0 = hw.store.stats()["launches"]
+    clk = Clocks(clocks_index) if clocks_index is not None else None
+    if clk:
+        clk.__enter__()
+        time.sleep(0.3)
+    dist_ctx.barrier()
+    torch.cuda.synchronize(hw.device)
+    t0 = torch.cuda.Event(enable_timing=True)
+    t1 = torch.cuda.Event(enable_timing=True)
+    t0.record(stream)
+    for k in range(steps):
+        hw.step(stream.cuda_stream, evs[k] if per_kernel else None)
+    t1.record(stream)
+    torch.cuda.synchronize(hw.device)
+    dist_ctx.barrier()
+    if clk:
+        clk.__exit__()
+    ms = t0.elapsed_time(t1)
+    launches = hw.store.stats()["launches"] - launches0
+    kern = None
+    if per_kernel:
+        put_ms = [a.elapsed_time(b) for e in evs for a, b in e["put"]]
+        get_ms = [a.elapsed_time(b) for e in evs for a, b in e["get"]]
+        kern = {"put_ms": statistics.mean(put_ms), "get_ms": statistics.mean(get_ms),
+                "put_bytes": hw.put_bytes / hw.requests, "get_bytes": hw.get_bytes / hw.requests,
+                "put_total_ms": sum(put_ms), "get_total_ms": sum(get_ms)}
+    return ms, launches, kern, (clk.summary() if clk else None)
+
+
+class Dist:
+    def __init__(self, n):
+        self.world = int(os.environ.get("WORLD_SIZE", "1"))
+        self.rank = int(os.environ.get("RANK", "0"))
+        self.local = int(os.environ.get("LOCAL_RANK", "0"))
+        self.on = self.world > 1
+        if self.on:
+            import torch.distributed as dist
+            self.dist = dist
+            dist.init_process_group("nccl" if os.environ.get("T2I_BENCH_GLOO") is None else "gloo")
+
+    def barrier(self):
+        if self.on:
+            self.dist.barrier()
+
+    def max(self, x: float) -> float:
+        if not self.on:
+            return x
+        import torch
+        t = torch.tensor([x], dtype=torch.float64, device=f"cuda:{self.local}" if torch.cuda.is_available() else "cpu")
+        self.dist.all_reduce(t, op=self.dist.ReduceOp.MAX)
+        return float(t.item())
+
+    def close(self):
+        if self.on:
+            self.dist.destroy_process_group()
+
+
+# ----------------------------------------------------------------------------- CPU (oracle)
+def oracle_sample(B: int, n_requests: int):
+    """The oracle as it stands on the host: put + get (latents cast) of
+    ``n_requests`` handoff requests (inputs of one request reused). Returns
+    (GB/s, seconds, bytes)."""
+    from oracle import OracleStore, PutItem
+
+    specs = W.handoff_specs(B)
+    arrs = W.handoff_request(0, 0, specs)
+    raw = [a.view(np.uint8).reshape(-1) for a in arrs]
+    ci = W.handoff_cast_index()
+    casts = [1 if j == ci else 0 for j in range(len(specs))]
+    store = OracleStore(W.HANDOFF["pool_bytes"], W.HANDOFF["page_bytes"])
+    payload = sum(sp.nbytes for sp in specs)
+    lat = specs[ci].nbytes
+    per_req = 2 * payload + 2 * (payload - lat) + 1.5 * lat
+    t = time.perf_counter()
+    ids_all = []
+    for _ in range(n_requests):
+        st, ids = store.put_batch([PutItem(x.size, x, sp.dtype_tag) for x, sp in zip(raw, specs)])
+        ids_all.append(ids)
+    for ids in ids_all:
+        store.get_batch(ids, casts)
+    for ids in ids_all:
+        store.free(ids)
+    dt = time.perf_counter() - t
+    return per_req * n_requests / dt / 1e9, dt, per_req * n_requests
+
+
+# ----------------------------------------------------------------------------- main
+def run_reference(args, dist_ctx):
+    if dist_ctx.rank != 0:
+        return
+    B = args.batch
+    n_req = 8
+    for _ in range(args.warmup):
+        oracle_sample(B, 1)
+    vals = []
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        v, dt, nb = oracle_sample(B, n_req)
+        vals.append((v, dt))
+    total_t = sum(dt for _, dt in vals)
+    total_b = sum(v * dt for v, dt in vals)
+    value = total_b / total_t
+    ms = 1e3 * total_t / len(vals)
+    line = {
+        "impl": "reference", "metric": METRIC, "value": round(value, 3), "unit": "GB/s", "n_gpus": args.gpus,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms, 3), "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "u8+f32->bf16", "data": "synthetic",
+        "config": {"workload": f"t2i handoff, B={B}, {n_req} requests per step (bounded sample of 64)",
+                   "pool_bytes": W.HANDOFF["pool_bytes"], "page_bytes": W.HANDOFF["page_bytes"]},
+        "cpu_baseline": {"value": round(value, 3), "unit": "GB/s", "cores": 1, "kind": "oracle",
+                         "sample": f"{n_req} of 64 requests per step, numpy oracle, single thread"},
+        "e2e": {"value": round(value, 3), "unit": "GB/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+        "wall_s": round(time.perf_counter() - t0, 2),
+    }
+    print(json.dumps(line), flush=True)
+
+
+def main():
+    args = parse()
+    dist_ctx = Dist(args.gpus)
+    if args.impl == "reference":
+        run_reference(args, dist_ctx)
+        dist_ctx.close()
+        return
+    import torch
+
+    from paper_2607_26566_gb300 import build as b
+
+    b.ensure_built()
+    device = torch.device("cuda", dist_ctx.local)
+    torch.cuda.set_device(device)
+    B = args.batch
+    hw = Handoff(B, args.requests, device)
+    ms, launches, kern, clocks = time_handoff(hw, args.steps, args.warmup, dist_ctx, per_kernel=True,
+                                              clocks_index=dist_ctx.local)
+    hw.verify()
+    ms_max = dist_ctx.max(ms)
+    total_bytes = hw.step_bytes * args.steps * dist_ctx.world
+    value = total_bytes / (ms_max * 1e-3) / 1e9
+    peak, peak_kind = peaks()
+
+    # dominant kernel: the one with more total time in the timed region
+    dom = "gather_get_kernel" if kern["get_total_ms"] >= kern["put_total_ms"] else "scatter_put_kernel"
+    k_ms = kern["get_ms"] if dom == "gather_get_kernel" else kern["put_ms"]
+    k_bytes = kern["get_bytes"] if dom == "gather_get_kernel" else kern["put_bytes"]
+    achieved = k_bytes / (k_ms * 1e-3) / 1e9
+    traffic = ncu_traffic(dom, f"handoff_B{B}_request")
+    roofline = {"bound": "hbm", "achieved": round(achieved, 1), "peak": peak, "unit": "GB/s",
+                "frac": round(achieved / peak, 4), "peak_kind": peak_kind,
+                "traffic": traffic,
+                "kernel": dom, "algorithmic_bytes_per_launch": k_bytes, "avg_launch_ms": round(k_ms, 5),
+                "other_kernel": {"name": "scatter_put_kernel" if dom == "gather_get_kernel" else "gather_get_kernel",
+                                 "achieved": round((kern["put_bytes"] / (kern["put_ms"] * 1e-3) / 1e9)
+                                                   if dom == "gather_get_kernel" else
+                                                   (kern["get_bytes"] / (kern["get_ms"] * 1e-3) / 1e9), 1)}}
+    del hw
+    torch.cuda.empty_cache()
+
+    sweep = {}
+    if args.sweep:
+        for Bs in (1, 4):
+            hs = Handoff(Bs, args.requests, device)
+            ms_s, _, _, _ = time_handoff(hs, max(3, args.steps // 2), args.warmup, dist_ctx, per_kernel=False)
+            sweep[f"B{Bs}"] = round(hs.step_bytes * max(3, args.steps // 2) / (ms_s * 1e-3) / 1e9, 1)
+            del hs
+            torch.cuda.empty_cache()
+
+    e2e = None
+    if not args.no_e2e:
+        he = Handoff(B, args.requests, device, host_buffers=True)
+        e_steps = max(2, min(args.steps, 3))
+        ms_e, _, _, _ = time_handoff(he, e_steps, 1, dist_ctx, per_kernel=False)
+        ms_e = dist_ctx.max(ms_e)
+        e2e = {"value": round(he.step_bytes * e_steps * dist_ctx.world / (ms_e * 1e-3) / 1e9, 2), "unit": "GB/s",
+               "h2d_bytes_per_step": int(he.h2d_bytes), "d2h_bytes_per_step": int(he.d2h_bytes),
+               "path": "t2i_put_batch / t2i_get_batch with pinned host sources and destinations"}
+        del he
+        torch.cuda.empty_cache()
+
+    cpu = None
+    if not args.no_cpu and dist_ctx.rank == 0:
+        v, dt, nb = oracle_sample(B, 16)
+        cpu = {"value": round(v, 3), "unit": "GB/s", "cores": 1, "kind": "oracle",
+               "sample": f"16 B={B} requests put + get (latents cast) by the numpy oracle, {dt:.1f} s"}
+
+    if dist_ctx.rank == 0:
+        line = {
+            "metric": METRIC, "value": round(value, 1), "unit": "GB/s", "n_gpus": dist_ctx.world,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms_max / args.steps, 4),
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "u8+f32->bf16",
+            "data": "synthetic",
+            "config": {"workload": f"t2i handoff, B={B}, {args.requests} requests in flight",
+                       "pool_bytes": W.HANDOFF["pool_bytes"], "page_bytes": W.HANDOFF["page_bytes"],
+                       "bytes_per_step": hw_bytes(B, args.requests), "l2": "inputs > L2 (no flush)",
+                       "parallelism": f"replicas x{dist_ctx.world}"},
+            "hbm_frac": round(value / dist_ctx.world / peak, 4), "hbm_frac_nominal_8tbs": round(value / dist_ctx.world / 8000.0, 4),
+            "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e, "gpu_launches": int(launches),
+            "clocks": clocks, "sweep": sweep or None,
+        }
+        print(json.dumps(line), flush=True)
+    dist_ctx.close()
+
+
+def hw_bytes(B, requests):
+    specs = W.handoff_specs(B)
+    payload = sum(sp.nbytes for sp in specs)
+    lat = specs[W.handoff_cast_index()].nbytes
+    return int((2 * payload + 2 * (payload - lat) + 1.5 * lat) * requests)
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,220 @@
+/*
+ * t2istore.h -- a paged tensor store in the spare HBM of one GPU (GB300, sm_103a).
+ *
+ * The store is the GPU-resident data plane of a serverless text-to-image
+ * system (arxiv 2607.26566, §5): model functions put intermediate tensors
+ * (text embeddings, latents, decoded images) and cached model or adapter
+ * weights into it, and get them back into their own buffers. The pool is one
+ * block of device memory that the caller owns (typically a PyTorch
+ * allocation); the store divides it into fixed pages and keeps the page
+ * tables, the object directory and the LRU order on the host. Bytes move only
+ * through the library's own CUDA kernels (and, for host sources on request,
+ * the copy engine), stream-ordered on the caller's stream.
+ *
+ * Conventions shared by every call:
+ *  - Every call returns a t2i_status; nothing aborts or prints.
+ *  - The caller owns the pool, every source and destination buffer and every
+ *    descriptor array. Descriptor arrays are read only during the call.
+ *  - Calls are asynchronous like cudaMemcpyAsync: a put's sources must stay
+ *    unchanged until the stream has passed the put; a get's destinations hold
+ *    the bytes once the stream has passed the get.
+ *  - All work of one store is ordered: a call on a stream other than the
+ *    previous call's waits (on the GPU, through an event) for that call's
+ *    work, so pages freed by one call are reused only by later work.
+ *  - Pointers are checked on the host before any launch (when
+ *    check_pointers = 1): a pointer the CUDA driver does not know, on another
+ *    device, or a range that runs past its allocation returns
+ *    T2I_ERR_INVALID, so a bad argument never reaches the GPU.
+ *  - A store may be used from several host threads; calls are serialised by
+ *    a lock inside the store.
+ */
+#ifndef T2ISTORE_H
+#define T2ISTORE_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* ---- status codes ------------------------------------------------------ */
+typedef int32_t t2i_status;
+#define T2I_OK 0
+#define T2I_ERR_INVALID 1   /* bad argument; nothing changed                     */
+#define T2I_ERR_NOSPACE 2   /* not enough pages even after eviction; nothing changed */
+#define T2I_ERR_NOT_FOUND 3 /* id never issued, or already freed                 */
+#define T2I_ERR_EVICTED 4   /* id was evicted to make room (put it again)        */
+#define T2I_ERR_CUDA 5      /* a CUDA call failed; see t2i_last_error            */
+
+/* Object ids: 1, 2, 3, ... in descriptor order, never reused; 0 is never an id. */
+typedef uint64_t t2i_id;
+
+typedef struct t2i_store t2i_store; /* opaque: a store over one pool          */
+typedef struct t2i_ctl t2i_ctl;     /* opaque: the host control core alone     */
+
+/* ---- configuration ------------------------------------------------------- */
+typedef struct t2i_store_config {
+    uint64_t pool_bytes;     /* bytes at pool_dev; the store uses floor(pool_bytes / page_bytes) pages */
+    uint64_t page_bytes;     /* power of two, 256 B ... 1 GiB                                   */
+    uint32_t h2d_mode;       /* puts from host memory: 0 = the put kernel reads pinned host memory
+                                directly (zero-copy over the host link); 1 = one copy-engine
+                                cudaMemcpyAsync per run of consecutive pages. Pageable (not
+                                pinned) host memory always takes the copy engine.               */
+    uint32_t check_pointers; /* 1 = check every user pointer range with the driver before launch
+                                (recommended); 0 = trust the caller                             */
+} t2i_store_config;
+
+/* ---- put ------------------------------------------------------------------
+ * One object to store. Ids are returned in descriptor order.
+ * §5.2: a producer writes its output into the store; §5.3: cached weights are
+ * evictable, least recently used model first, higher layers first.        */
+typedef struct t2i_put_desc {
+    const void* src;      /* nbytes to copy: device memory of the store's device, or host memory
+                             when src_is_host = 1. NULL reserves pages and copies nothing (the
+                             object's bytes are undefined until overwritten by nobody: a
+                             placeholder that only takes capacity).                          */
+    uint64_t nbytes;      /* object size; 0 is allowed (no pages)                            */
+    uint32_t src_is_host; /* 1 = src is host memory (pinned or pageable)                      */
+    uint32_t dtype_tag;   /* opaque tag kept in the directory                                 */
+    uint64_t group;       /* LRU group: one model or one adapter set                          */
+    uint32_t order;       /* layer index inside the group; the highest is evicted first        */
+    uint32_t evictable;   /* 1 = cached weights (may be evicted); 0 = intermediate (never)      */
+} t2i_put_desc;
+
+/* ---- get ------------------------------------------------------------------
+ * Copies an object into a consumer buffer (§5.2: the consumer pulls a
+ * produced tensor into its own memory), optionally casting fp32 -> bf16.  */
+typedef struct t2i_get_desc {
+    t2i_id id;
+    void* dst;            /* device memory of the store's device, or pinned host memory      */
+    uint64_t dst_bytes;   /* capacity at dst: >= nbytes, or >= nbytes / 2 with cast = 1       */
+    uint32_t cast;        /* 0 = bytes as stored; 1 = the object is little-endian fp32 and dst
+                             receives bf16, round to nearest even (NaN -> quiet NaN with the
+                             sign kept: 0x7FC0 | sign << 15); needs nbytes % 4 == 0 and a
+                             2-byte aligned dst                                               */
+    uint32_t reserved;    /* must be 0                                                        */
+} t2i_get_desc;
+
+/* ---- compaction moves ------------------------------------------------------ */
+typedef struct t2i_move {
+    uint32_t src_page;    /* live page at or above the limit                                  */
+    uint32_t dst_page;    /* lowest free page below the limit                                 */
+    uint64_t valid_bytes; /* bytes of the object in that page (only these are copied)          */
+} t2i_move;
+
+/* ---- introspection ----------------------------------------------------------- */
+typedef struct t2i_stats {
+    uint64_t total_pages, limit_pages, used_pages, free_pages, live_objects;
+    uint64_t bytes_put, bytes_got, puts, gets, misses, evictions;
+    uint64_t pages_moved, bytes_moved;
+    uint64_t launches;   /* kernels launched by the store                                    */
+    uint64_t h2d_copies; /* copy-engine copies issued for host sources                        */
+} t2i_stats;
+
+typedef struct t2i_object_info {
+    uint64_t nbytes;
+    uint64_t group;
+    uint32_t dtype_tag;
+    uint32_t order;
+    uint32_t evictable;
+    uint32_t n_pages;
+} t2i_object_info;
+
+/* =========================================================================
+ * Store: the pool, the host control core and the CUDA kernels.
+ * ========================================================================= */
+
+/* Creates a store over [pool_dev, pool_dev + pool_bytes) on CUDA device
+ * `device`. pool_dev must be device memory of that device, 256-byte aligned.
+ * The store never frees pool_dev. Errors: INVALID (geometry, pointer),
+ * CUDA (device query failed). On error *out is NULL and t2i_last_error(NULL)
+ * describes it.                                                             */
+t2i_status t2i_store_create(void* pool_dev, const t2i_store_config* cfg, int device, t2i_store** out);
+
+/* Frees the store's host state and events after waiting for its last work.
+ * Does not free the pool. NULL is accepted.                                 */
+t2i_status t2i_store_destroy(t2i_store* store);
+
+/* Stores n objects (paper §5.2 "producer writes its output", §5.3 eviction).
+ * All-or-nothing: pages for the whole batch are taken from the free stack,
+ * evicting least-recently-used evictable objects of groups not named in this
+ * batch (highest `order`, then highest id, first) until the batch fits.
+ * Returns NOSPACE (and evicts nothing) if even that is not enough, INVALID
+ * for a bad descriptor; out_ids[i] receives the id of descs[i] (n ids).
+ * The copy is one kernel launch per batch (more only when the descriptors
+ * exceed one launch's parameter space). On CUDA the batch is not stored;
+ * evictions it made stand.                                                   */
+t2i_status t2i_put_batch(t2i_store* store, const t2i_put_desc* descs, uint32_t n, t2i_id* out_ids,
+                         void* cuda_stream);
+
+/* Copies n objects into their destinations (paper §5.2 "consumer pulls").
+ * Every item is validated first; per_item (nullable, n entries) receives
+ * OK / NOT_FOUND / EVICTED / INVALID per item. If any item fails, the call
+ * returns the first failing status in descriptor order and writes nothing.
+ * The same id may appear more than once. Objects reserved with src = NULL
+ * return whatever their pages hold.                                          */
+t2i_status t2i_get_batch(t2i_store* store, const t2i_get_desc* descs, uint32_t n, t2i_status* per_item,
+                         void* cuda_stream);
+
+/* Returns the pages of n objects to the free stack (paper §5.3: data is
+ * reclaimed when no consumer needs it). Host-only: stream order makes reuse
+ * safe. A repeated id is INVALID; an unknown id is NOT_FOUND; in both cases
+ * nothing is freed. An evicted id is accepted and forgotten.                 */
+t2i_status t2i_free(t2i_store* store, const t2i_id* ids, uint32_t n);
+
+/* Shrinks (or regrows) the usable pool to limit_bytes (a multiple of
+ * page_bytes, at most the pool): live pages at or above the limit move, in
+ * ascending order, to the lowest free pages below it (one kernel; only the
+ * valid bytes of each page are copied) and the page tables are remapped.
+ * NOSPACE if more than limit_bytes / page_bytes pages are in use. After the
+ * stream has passed this call, [pool + limit_bytes, pool + pool_bytes) is
+ * not touched by the store until a larger limit is set. pages_moved is
+ * nullable. (No counterpart in the paper: it answers the fixed-size arena
+ * problem of §5.3.)                                                          */
+t2i_status t2i_compact(t2i_store* store, uint64_t limit_bytes, void* cuda_stream, uint64_t* pages_moved);
+
+t2i_status t2i_store_stats(const t2i_store* store, t2i_stats* out);
+
+/* The store's host control core (read-only: the t2i_ctl_* queries below
+ * accept it; the mutating t2i_ctl_* calls refuse it with INVALID).          */
+const t2i_ctl* t2i_store_ctl(const t2i_store* store);
+
+/* Message of the last failed call on this store (or, for NULL, of the last
+ * failed t2i_store_create / t2i_ctl_create on this thread). Never NULL.      */
+const char* t2i_last_error(const t2i_store* store);
+
+/* =========================================================================
+ * Control core: page allocator, directory, LRU and compaction planner,
+ * without device memory. The same code runs inside every store; alone it
+ * plans layouts on the host and is what the host-only tests drive.
+ * ========================================================================= */
+
+/* total_pages <= 2^32 - 1, page_bytes > 0.                                  */
+t2i_status t2i_ctl_create(uint64_t total_pages, uint64_t page_bytes, t2i_ctl** out);
+t2i_status t2i_ctl_destroy(t2i_ctl* ctl);
+/* As t2i_put_batch, without copying (src and src_is_host are ignored).      */
+t2i_status t2i_ctl_put(t2i_ctl* ctl, const t2i_put_desc* descs, uint32_t n, t2i_id* out_ids);
+/* As t2i_get_batch's validation and LRU update (dst/dst_bytes ignored).     */
+t2i_status t2i_ctl_get(t2i_ctl* ctl, const t2i_get_desc* descs, uint32_t n, t2i_status* per_item);
+t2i_status t2i_ctl_free(t2i_ctl* ctl, const t2i_id* ids, uint32_t n);
+/* As t2i_compact's planning and remap. moves (nullable) receives the moves
+ * in order if cap is large enough; otherwise INVALID with *n_moves set to
+ * the number needed and nothing changed.                                    */
+t2i_status t2i_ctl_compact(t2i_ctl* ctl, uint64_t limit_bytes, t2i_move* moves, uint64_t cap, uint64_t* n_moves);
+
+/* Queries (accept a store's control core). pages receives up to cap page
+ * numbers of the object in page-list order; info->n_pages is the full count. */
+t2i_status t2i_ctl_object(const t2i_ctl* ctl, t2i_id id, t2i_object_info* info, uint32_t* pages, uint64_t cap);
+/* The free stack from bottom to top (the top pops first); *n = its size.     */
+t2i_status t2i_ctl_free_pages(const t2i_ctl* ctl, uint32_t* out, uint64_t cap, uint64_t* n);
+/* Ids evicted by the last put, in eviction order; *n = their number.         */
+t2i_status t2i_ctl_last_evictions(const t2i_ctl* ctl, t2i_id* out, uint64_t cap, uint64_t* n);
+t2i_status t2i_ctl_stats(const t2i_ctl* ctl, t2i_stats* out);
+const char* t2i_ctl_last_error(const t2i_ctl* ctl);
+
+#ifdef __cplusplus
+} /* extern "C" */
+#endif
+
+#endif /* T2ISTORE_H */

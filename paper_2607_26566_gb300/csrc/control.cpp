@@ -1,0 +1,358 @@
+// Host control core: see control.hpp for the rules it implements.
+#include "control.hpp"
+
+#include <algorithm>
+#include <string>
+
+namespace t2i {
+
+// ---------------------------------------------------------------- IdTable
+uintptr_t IdTable::get(uint64_t id) const {
+    const uint64_t leaf = id >> kLeafBits;
+    if (leaf >= leaves_.size() || !leaves_[leaf]) return 0;
+    return leaves_[leaf]->slot[id & (kLeafSize - 1)];
+}
+
+void IdTable::set(uint64_t id, uintptr_t v, uint64_t /*next_id*/) {
+    const uint64_t leaf = id >> kLeafBits;
+    if (leaf >= leaves_.size()) leaves_.resize(leaf + 1);
+    if (!leaves_[leaf]) leaves_[leaf].reset(new Leaf());
+    Leaf* L = leaves_[leaf].get();
+    uintptr_t& s = L->slot[id & (kLeafSize - 1)];
+    if (s == 0) L->used++;
+    s = v;
+}
+
+void IdTable::clear(uint64_t id, uint64_t next_id) {
+    const uint64_t leaf = id >> kLeafBits;
+    if (leaf >= leaves_.size() || !leaves_[leaf]) return;
+    Leaf* L = leaves_[leaf].get();
+    uintptr_t& s = L->slot[id & (kLeafSize - 1)];
+    if (s != 0) {
+        s = 0;
+        L->used--;
+    }
+    // every id of the leaf has been issued and none is live or evicted: no
+    // lookup can find anything in it any more
+    if (L->used == 0 && (leaf + 1) * kLeafSize <= next_id) leaves_[leaf].reset();
+}
+
+// ---------------------------------------------------------------- Control
+Control::Control(uint64_t total_pages, uint64_t page_bytes)
+    : P_(page_bytes), total_pages_(total_pages), limit_pages_(total_pages) {
+    free_.reserve(total_pages);
+    for (uint64_t p = total_pages; p-- > 0;) free_.push_back(static_cast<uint32_t>(p));
+}
+
+Control::~Control() {
+    for (Object* o : live_) delete o;
+}
+
+Group* Control::group_for(uint64_t key) {
+    auto it = groups_.find(key);
+    if (it != groups_.end()) return it->second.get();
+    auto g = std::make_unique<Group>();
+    g->key = key;
+    Group* raw = g.get();
+    groups_.emplace(key, std::move(g));
+    return raw;
+}
+
+void Control::maybe_drop_group(Group* g) {
+    if (g->n_objects == 0 && g->victims.empty() && g->rec_key == 0 && g->epoch != epoch_) groups_.erase(g->key);
+}
+
+void Control::touch(Object* o) {
+    Group* g = o->group;
+    g->last = ++clock_;
+    if (g->epoch != epoch_) {
+        g->epoch = epoch_;
+        touched_.push_back(g);
+    }
+}
+
+void Control::flush_touches() {
+    for (Group* g : touched_) {
+        if (g->victims.empty()) continue;
+        if (g->rec_key) recency_.erase({g->rec_key, g});
+        recency_.insert({g->last, g});
+        g->rec_key = g->last;
+    }
+    touched_.clear();
+    ++epoch_;
+}
+
+void Control::release(Object* o, bool evicted) {
+    const uint64_t np = o->pages.size();
+    for (uint32_t p : o->pages) free_.push_back(p);
+    used_pages_ -= np;
+    Group* g = o->group;
+    g->n_objects--;
+    if (o->evictable) {
+        g->victims.erase({o->order, o->id});
+        g->evictable_pages -= np;
+        evictable_pages_ -= np;
+        if (g->victims.empty() && g->rec_key) {
+            recency_.erase({g->rec_key, g});
+            g->rec_key = 0;
+        }
+    }
+    const size_t i = o->live_index;
+    live_[i] = live_.back();
+    live_[i]->live_index = i;
+    live_.pop_back();
+    if (evicted)
+        ids_.set(o->id, IdTable::kEvicted, next_id_);
+    else
+        ids_.clear(o->id, next_id_);
+    delete o;
+    maybe_drop_group(g);
+}
+
+uint64_t Control::live_pages_at_or_above(uint64_t limit) const {
+    uint64_t k = 0;
+    for (const Object* o : live_)
+        for (uint32_t p : o->pages) k += p >= limit;
+    return k;
+}
+
+const Object* Control::find(uint64_t id) const {
+    const uintptr_t v = ids_.get(id);
+    return v > IdTable::kEvicted ? reinterpret_cast<const Object*>(v) : nullptr;
+}
+
+t2i_status Control::put(const t2i_put_desc* descs, uint32_t n, t2i_id* ids, std::vector<const Object*>* created) {
+    last_evictions_.clear();
+    if (created) created->clear();
+    if (n == 0) return T2I_OK;
+    if (!descs || !ids) {
+        err_ = "put: null descriptor or id array";
+        return T2I_ERR_INVALID;
+    }
+    uint64_t demand = 0;
+    std::vector<uint64_t> pinned;
+    pinned.reserve(n);
+    for (uint32_t i = 0; i < n; ++i) {
+        const uint64_t np = pages_for(descs[i].nbytes);
+        if (np > limit_pages_ || demand + np > limit_pages_) {
+            err_ = "put: the batch needs more pages than the store has";
+            return T2I_ERR_NOSPACE;
+        }
+        demand += np;
+        pinned.push_back(descs[i].group);
+    }
+    std::sort(pinned.begin(), pinned.end());
+    pinned.erase(std::unique(pinned.begin(), pinned.end()), pinned.end());
+
+    if (demand > free_.size()) {
+        uint64_t avail = evictable_pages_;
+        for (uint64_t key : pinned) {
+            auto it = groups_.find(key);
+            if (it != groups_.end()) avail -= it->second->evictable_pages;
+        }
+        if (free_.size() + avail < demand) {
+            err_ = "put: not enough free pages even after evicting every allowed object";
+            return T2I_ERR_NOSPACE;
+        }
+        auto it = recency_.begin();
+        while (free_.size() < demand && it != recency_.end()) {
+            Group* g = it->second;
+            auto next = std::next(it);
+            if (!std::binary_search(pinned.begin(), pinned.end(), g->key)) {
+                while (free_.size() < demand) {
+                    auto v = g->victims.begin();
+                    const bool last = std::next(v) == g->victims.end();
+                    Object* o = reinterpret_cast<Object*>(ids_.get(v->second));
+                    last_evictions_.push_back(o->id);
+                    counters_.evictions++;
+                    release(o, true);  // may drop g once its last victim is gone
+                    if (last) break;
+                }
+            }
+            it = next;
+        }
+    }
+
+    for (uint32_t i = 0; i < n; ++i) {
+        const t2i_put_desc& d = descs[i];
+        Object* o = new Object();
+        o->id = next_id_++;
+        o->nbytes = d.nbytes;
+        o->dtype_tag = d.dtype_tag;
+        o->order = d.order;
+        o->evictable = d.evictable != 0;
+        o->group = group_for(d.group);
+        const uint64_t np = pages_for(d.nbytes);
+        o->pages.resize(np);
+        for (uint64_t j = 0; j < np; ++j) {
+            o->pages[j] = free_.back();
+            free_.pop_back();
+        }
+        used_pages_ += np;
+        Group* g = o->group;
+        g->n_objects++;
+        if (o->evictable) {
+            g->victims.insert({o->order, o->id});
+            g->evictable_pages += np;
+            evictable_pages_ += np;
+        }
+        o->live_index = live_.size();
+        live_.push_back(o);
+        ids_.set(o->id, reinterpret_cast<uintptr_t>(o), next_id_);
+        touch(o);
+        counters_.puts++;
+        counters_.bytes_put += d.nbytes;
+        ids[i] = o->id;
+        if (created) created->push_back(o);
+    }
+    flush_touches();
+    return T2I_OK;
+}
+
+void Control::rollback_put(const t2i_id* ids, uint32_t n) {
+    for (uint32_t i = 0; i < n; ++i) {
+        Object* o = const_cast<Object*>(find(ids[i]));
+        if (!o) continue;
+        counters_.puts--;
+        counters_.bytes_put -= o->nbytes;
+        release(o, false);
+    }
+}
+
+t2i_status Control::get(const t2i_get_desc* descs, uint32_t n, t2i_status* per_item,
+                        std::vector<const Object*>* objs) {
+    if (objs) objs->assign(n, nullptr);
+    if (n == 0) return T2I_OK;
+    if (!descs) {
+        err_ = "get: null descriptor array";
+        return T2I_ERR_INVALID;
+    }
+    t2i_status first = T2I_OK;
+    uint32_t first_i = 0;
+    for (uint32_t i = 0; i < n; ++i) {
+        const t2i_get_desc& d = descs[i];
+        t2i_status st = T2I_OK;
+        if (d.cast > 1 || d.reserved != 0) {
+            st = T2I_ERR_INVALID;
+        } else {
+            const uintptr_t v = ids_.get(d.id);
+            if (v == 0) {
+                st = T2I_ERR_NOT_FOUND;
+            } else if (v == IdTable::kEvicted) {
+                st = T2I_ERR_EVICTED;
+                counters_.misses++;
+            } else {
+                const Object* o = reinterpret_cast<const Object*>(v);
+                if (d.cast == 1 && (o->nbytes % 4) != 0) st = T2I_ERR_INVALID;
+                if (objs) (*objs)[i] = o;
+            }
+        }
+        if (per_item) per_item[i] = st;
+        if (st != T2I_OK && first == T2I_OK) {
+            first = st;
+            first_i = i;
+        }
+    }
+    if (first != T2I_OK) {
+        static const char* what[] = {"ok", "invalid descriptor (cast needs nbytes % 4 == 0)", "no space",
+                                     "id not found", "id was evicted", "cuda"};
+        err_ = "get: item " + std::to_string(first_i) + ": " + what[first];
+        return first;
+    }
+    for (uint32_t i = 0; i < n; ++i) {
+        Object* o = reinterpret_cast<Object*>(ids_.get(descs[i].id));
+        touch(o);
+        counters_.gets++;
+        counters_.bytes_got += o->nbytes;
+    }
+    flush_touches();
+    return T2I_OK;
+}
+
+t2i_status Control::free(const t2i_id* ids, uint32_t n) {
+    if (n == 0) return T2I_OK;
+    if (!ids) {
+        err_ = "free: null id array";
+        return T2I_ERR_INVALID;
+    }
+    std::vector<uint64_t> sorted(ids, ids + n);
+    std::sort(sorted.begin(), sorted.end());
+    if (std::adjacent_find(sorted.begin(), sorted.end()) != sorted.end()) {
+        err_ = "free: an id appears twice";
+        return T2I_ERR_INVALID;
+    }
+    for (uint32_t i = 0; i < n; ++i) {
+        if (ids_.get(ids[i]) == 0) {
+            err_ = "free: id " + std::to_string(ids[i]) + " not found";
+            return T2I_ERR_NOT_FOUND;
+        }
+    }
+    for (uint32_t i = 0; i < n; ++i) {
+        const uintptr_t v = ids_.get(ids[i]);
+        if (v == IdTable::kEvicted)
+            ids_.clear(ids[i], next_id_);
+        else
+            release(reinterpret_cast<Object*>(v), false);
+    }
+    return T2I_OK;
+}
+
+t2i_status Control::compact(uint64_t limit_bytes, std::vector<t2i_move>* moves) {
+    moves->clear();
+    if (limit_bytes % P_ != 0 || limit_bytes / P_ > total_pages_) {
+        err_ = "compact: the limit must be a multiple of the page size and at most the pool";
+        return T2I_ERR_INVALID;
+    }
+    const uint64_t limit = limit_bytes / P_;
+    if (used_pages_ > limit) {
+        err_ = "compact: more pages are in use than the limit holds";
+        return T2I_ERR_NOSPACE;
+    }
+    struct Tail {
+        uint32_t page;
+        Object* o;
+        uint32_t idx;
+    };
+    std::vector<uint8_t> used(limit, 0);
+    std::vector<Tail> tail;
+    for (Object* o : live_) {
+        for (uint32_t j = 0; j < o->pages.size(); ++j) {
+            const uint32_t p = o->pages[j];
+            if (p < limit)
+                used[p] = 1;
+            else
+                tail.push_back({p, o, j});
+        }
+    }
+    std::sort(tail.begin(), tail.end(), [](const Tail& a, const Tail& b) { return a.page < b.page; });
+    moves->reserve(tail.size());
+    uint64_t scan = 0;
+    uint64_t moved_bytes = 0;
+    for (const Tail& t : tail) {
+        while (used[scan]) ++scan;  // used_pages_ <= limit guarantees a free page
+        const uint32_t dst = static_cast<uint32_t>(scan);
+        used[scan] = 1;
+        const uint64_t valid = std::min<uint64_t>(P_, t.o->nbytes - uint64_t(t.idx) * P_);
+        t.o->pages[t.idx] = dst;
+        moves->push_back({t.page, dst, valid});
+        moved_bytes += valid;
+    }
+    free_.clear();
+    for (uint64_t p = limit; p-- > 0;)
+        if (!used[p]) free_.push_back(static_cast<uint32_t>(p));
+    limit_pages_ = limit;
+    counters_.pages_moved += tail.size();
+    counters_.bytes_moved += moved_bytes;
+    return T2I_OK;
+}
+
+void Control::stats(t2i_stats* out) const {
+    *out = counters_;
+    out->total_pages = total_pages_;
+    out->limit_pages = limit_pages_;
+    out->used_pages = used_pages_;
+    out->free_pages = free_.size();
+    out->live_objects = live_.size();
+}
+
+}  // namespace t2i

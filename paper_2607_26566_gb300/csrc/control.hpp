@@ -1,0 +1,149 @@
+// Host control core of the paged tensor store: page allocator, object
+// directory, per-group LRU and compaction planner. Plain C++17, no CUDA.
+//
+// The paper's data plane keeps a fixed-size arena per executor managed by a
+// buddy allocator (§5.2) and a Layer Lookup Table that maps a model's logical
+// layers to tensor objects and their physical memory (§5.3, "How does it
+// work?"). Here the arena is cut into fixed pages and the lookup table is the
+// directory id -> {size, tags, page list}. Eviction follows §5.3: least
+// recently used model first, its layers in reverse order, until the demand is
+// met. Where the paper is silent the rules are:
+//   - free pages form a LIFO stack; page 0 pops first on a new store; a put
+//     pops its pages one at a time, objects in descriptor order; a free pushes
+//     an object's pages back in page-list order;
+//   - ids are 1, 2, 3, ... in descriptor order and never reused;
+//   - recency is per group, stamped once per object put or got, in
+//     descriptor order; victims: least recent group first, then the highest
+//     `order`, then the highest id; groups named by the put are exempt, so are
+//     non-evictable objects; a put that cannot be satisfied evicts nothing;
+//   - compaction to `limit` pages moves the live pages numbered >= limit, in
+//     ascending order, to the lowest free pages below limit, then rebuilds the
+//     free stack from the free pages below limit so the lowest pops first.
+#pragma once
+
+#include <cstdint>
+#include <memory>
+#include <set>
+#include <string>
+#include <unordered_map>
+#include <utility>
+#include <vector>
+
+#include "t2istore.h"
+
+namespace t2i {
+
+struct Group;
+
+struct Object {
+    uint64_t id = 0;
+    uint64_t nbytes = 0;
+    uint32_t dtype_tag = 0;
+    uint32_t order = 0;
+    bool evictable = false;
+    Group* group = nullptr;
+    size_t live_index = 0;          // position in Control::live_
+    std::vector<uint32_t> pages;    // page list, in object byte order
+};
+
+struct Group {
+    uint64_t key = 0;
+    uint64_t last = 0;              // recency stamp of the last touch
+    uint64_t rec_key = 0;           // stamp under which it sits in the recency set; 0 = absent
+    uint64_t n_objects = 0;
+    uint64_t evictable_pages = 0;
+    uint64_t epoch = 0;             // batch marker for de-duplicating touches
+    // evictable objects, eviction order first: highest order, then highest id
+    std::set<std::pair<uint32_t, uint64_t>, std::greater<std::pair<uint32_t, uint64_t>>> victims;
+};
+
+// id -> object, or the "evicted" tombstone; two-level table over the dense
+// id space whose leaves are released once every id in them is gone.
+class IdTable {
+  public:
+    static constexpr uintptr_t kEvicted = 1;
+    uintptr_t get(uint64_t id) const;
+    void set(uint64_t id, uintptr_t v, uint64_t next_id);
+    void clear(uint64_t id, uint64_t next_id);
+
+  private:
+    static constexpr int kLeafBits = 12;
+    static constexpr uint64_t kLeafSize = uint64_t(1) << kLeafBits;
+    struct Leaf {
+        uintptr_t slot[kLeafSize] = {};
+        uint64_t used = 0;
+    };
+    std::vector<std::unique_ptr<Leaf>> leaves_;
+};
+
+
+class Control {
+  public:
+    Control(uint64_t total_pages, uint64_t page_bytes);
+    ~Control();
+    Control(const Control&) = delete;
+    Control& operator=(const Control&) = delete;
+
+    uint64_t page_bytes() const { return P_; }
+    uint64_t total_pages() const { return total_pages_; }
+    uint64_t limit_pages() const { return limit_pages_; }
+    uint64_t used_pages() const { return used_pages_; }
+    uint64_t pages_for(uint64_t nbytes) const { return nbytes / P_ + (nbytes % P_ != 0); }
+
+    // put: validates, evicts, allocates and commits. On success ids[i] and
+    // created[i] (if non-null) describe descs[i].
+    t2i_status put(const t2i_put_desc* descs, uint32_t n, t2i_id* ids, std::vector<const Object*>* created);
+    // Undo the put of freshly created objects (after a failed launch).
+    void rollback_put(const t2i_id* ids, uint32_t n);
+    // get: validates every item (per_item nullable), then stamps recency.
+    // objs[i] receives the object of descs[i] on success. dst fields are not
+    // looked at here.
+    t2i_status get(const t2i_get_desc* descs, uint32_t n, t2i_status* per_item, std::vector<const Object*>* objs);
+    t2i_status free(const t2i_id* ids, uint32_t n);
+    // compact: plans, remaps and returns the moves (always filled).
+    t2i_status compact(uint64_t limit_bytes, std::vector<t2i_move>* moves);
+
+    uint64_t live_pages_at_or_above(uint64_t limit) const;
+    const Object* find(uint64_t id) const;
+    bool is_evicted(uint64_t id) const { return ids_.get(id) == IdTable::kEvicted; }
+    const std::vector<uint32_t>& free_stack() const { return free_; }
+    const std::vector<t2i_id>& last_evictions() const { return last_evictions_; }
+    void stats(t2i_stats* out) const;
+    t2i_stats& counters() { return counters_; }
+
+    const std::string& error() const { return err_; }
+    void set_error(std::string e) { err_ = std::move(e); }
+
+  private:
+    Group* group_for(uint64_t key);
+    void maybe_drop_group(Group* g);
+    void touch(Object* o);
+    void flush_touches();
+    void release(Object* o, bool evicted);
+
+    uint64_t P_;
+    uint64_t total_pages_;
+    uint64_t limit_pages_;
+    uint64_t used_pages_ = 0;
+    uint64_t evictable_pages_ = 0;
+    uint64_t next_id_ = 1;
+    uint64_t clock_ = 0;
+    uint64_t epoch_ = 1;            // groups start at epoch 0, so the first batch is new
+    std::vector<uint32_t> free_;   // free page stack; back() is the top
+    IdTable ids_;
+    std::vector<Object*> live_;
+    std::unordered_map<uint64_t, std::unique_ptr<Group>> groups_;
+    std::set<std::pair<uint64_t, Group*>> recency_;   // groups holding evictable objects
+    std::vector<Group*> touched_;
+    std::vector<t2i_id> last_evictions_;
+    t2i_stats counters_{};
+    std::string err_;
+};
+
+}  // namespace t2i
+
+// The opaque C handle around a control core.
+struct t2i_ctl {
+    t2i::Control* core;
+    bool owned;      // false: borrowed from a store (queries only)
+};

@@ -1,0 +1,649 @@
+// The store: host control core + pointer checks + kernel launches, and the
+// t2i_store / t2i_put_batch / t2i_get_batch / t2i_free / t2i_compact C ABI.
+#include <cuda.h>
+#include <cuda_runtime.h>
+
+#include <algorithm>
+#include <cstring>
+#include <mutex>
+#include <new>
+#include <string>
+#include <vector>
+
+#include "common.hpp"
+#include "control.hpp"
+#include "kernels.cuh"
+
+namespace t2i {
+namespace {
+
+// ------------------------------------------------------------------ driver
+// Pointer attributes come from the driver API, fetched through the runtime
+// so that the library does not link libcuda (it loads on machines without
+// a driver, where only the t2i_ctl_* calls are usable).
+using PFN_getAttrs = CUresult (*)(unsigned int, CUpointer_attribute*, void**, CUdeviceptr);
+
+PFN_getAttrs driver_get_attrs() {
+    static PFN_getAttrs fn = []() -> PFN_getAttrs {
+        void* p = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuPointerGetAttributes", &p, 12000, cudaEnableDefault, &q) != cudaSuccess ||
+            q != cudaDriverEntryPointSuccess)
+            return nullptr;
+        return reinterpret_cast<PFN_getAttrs>(p);
+    }();
+    return fn;
+}
+
+enum class MemKind { Unknown, Device, Host, Managed };
+
+struct Range {
+    uint64_t start = 0, end = 0;  // [start, end)
+    MemKind kind = MemKind::Unknown;
+    int device = -1;
+    uint64_t dev_base = 0;  // device-visible address of `start` (host memory)
+};
+
+// Queries the allocation that holds p. false if the driver call failed.
+bool query_range(const void* p, Range* r) {
+    PFN_getAttrs fn = driver_get_attrs();
+    if (!fn) return false;
+    CUpointer_attribute attrs[6] = {CU_POINTER_ATTRIBUTE_MEMORY_TYPE,     CU_POINTER_ATTRIBUTE_DEVICE_ORDINAL,
+                                    CU_POINTER_ATTRIBUTE_RANGE_START_ADDR, CU_POINTER_ATTRIBUTE_RANGE_SIZE,
+                                    CU_POINTER_ATTRIBUTE_IS_MANAGED,       CU_POINTER_ATTRIBUTE_DEVICE_POINTER};
+    unsigned int mtype = 0;
+    int ordinal = -1;
+    CUdeviceptr start = 0;
+    size_t size = 0;
+    int managed = 0;
+    CUdeviceptr devptr = 0;
+    void* data[6] = {&mtype, &ordinal, &start, &size, &managed, &devptr};
+    if (fn(6, attrs, data, reinterpret_cast<CUdeviceptr>(p)) != CUDA_SUCCESS) return false;
+    r->start = start;
+    r->end = start + size;
+    r->device = ordinal;
+    if (managed)
+        r->kind = MemKind::Managed;
+    else if (mtype == CU_MEMORYTYPE_DEVICE)
+        r->kind = MemKind::Device;
+    else if (mtype == CU_MEMORYTYPE_HOST)
+        r->kind = MemKind::Host;
+    else
+        r->kind = MemKind::Unknown;
+    // device-visible address of the range start (same as the host address
+    // under unified addressing)
+    r->dev_base = devptr ? uint64_t(devptr) - (reinterpret_cast<uint64_t>(p) - start) : start;
+    if (r->kind == MemKind::Unknown) r->start = r->end = 0;
+    return true;
+}
+
+struct DeviceGuard {
+    int prev = -1;
+    bool switched = false;
+    explicit DeviceGuard(int dev) {
+        if (cudaGetDevice(&prev) == cudaSuccess && prev != dev) switched = cudaSetDevice(dev) == cudaSuccess;
+    }
+    ~DeviceGuard() {
+        if (switched) cudaSetDevice(prev);
+    }
+};
+
+int log2_exact(uint64_t v) {
+    int s = 0;
+    while ((uint64_t(1) << s) < v) ++s;
+    return (uint64_t(1) << s) == v ? s : -1;
+}
+
+}  // namespace
+
+// -------------------------------------------------------------------- Store
+class Store {
+  public:
+    Store(void* pool, const t2i_store_config& cfg, int device)
+        : pool_(reinterpret_cast<uint64_t>(pool)), cfg_(cfg), device_(device),
+          ctl_(cfg.pool_bytes / cfg.page_bytes, cfg.page_bytes) {
+        handle_.core = &ctl_;
+        handle_.owned = false;
+        page_shift_ = log2_exact(cfg.page_bytes);
+        unit_shift_ = std::min<uint32_t>(page_shift_, kUnitShiftMax);
+    }
+    ~Store() {
+        if (order_ev_) {
+            if (have_last_) {
+                cudaEventRecord(order_ev_, last_stream_);
+                cudaEventSynchronize(order_ev_);
+            }
+            cudaEventDestroy(order_ev_);
+        }
+    }
+
+    t2i_status init(std::string* err) {
+        DeviceGuard g(device_);
+        int sms = 0;
+        if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, device_) != cudaSuccess || sms <= 0) {
+            *err = "cannot query the device";
+            return T2I_ERR_CUDA;
+        }
+        // persistent grids: resident CTAs per SM x SMs, per kernel
+        const void* fns[3][2] = {
+            {reinterpret_cast<const void*>(scatter_put_kernel<kBlobLarge, false>),
+             reinterpret_cast<const void*>(scatter_put_kernel<kBlobLarge, true>)},
+            {reinterpret_cast<const void*>(gather_get_kernel<kBlobLarge, false>),
+             reinterpret_cast<const void*>(gather_get_kernel<kBlobLarge, true>)},
+            {reinterpret_cast<const void*>(compact_move_kernel<kBlobLarge>),
+             reinterpret_cast<const void*>(compact_move_kernel<kBlobLarge>)}};
+        for (int m = 0; m < 3; ++m)
+            for (int g = 0; g < 2; ++g) {
+                int occ = 0;
+                cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, fns[m][g], kThreads, 0);
+                max_ctas_[m][g] = sms * (occ > 0 ? occ : 1);
+            }
+        if (cudaEventCreateWithFlags(&order_ev_, cudaEventDisableTiming) != cudaSuccess) {
+            *err = "cannot create an event";
+            return T2I_ERR_CUDA;
+        }
+        return T2I_OK;
+    }
+
+    std::mutex mu;
+    t2i_ctl* ctl_handle() { return &handle_; }
+    Control& ctl() { return ctl_; }
+    const std::string& error() const { return err_; }
+
+    t2i_status put(const t2i_put_desc* descs, uint32_t n, t2i_id* ids, cudaStream_t stream);
+    t2i_status get(const t2i_get_desc* descs, uint32_t n, t2i_status* per_item, cudaStream_t stream);
+    t2i_status free(const t2i_id* ids, uint32_t n) {
+        t2i_status st = ctl_.free(ids, n);
+        if (st != T2I_OK) err_ = ctl_.error();
+        return st;
+    }
+    t2i_status compact(uint64_t limit_bytes, cudaStream_t stream, uint64_t* moved);
+
+  private:
+    // ---- pointer checks (per call cache of the last allocation seen)
+    t2i_status check_user(const void* p, uint64_t n, bool want_write, bool is_host_flag, uint64_t* dev_addr,
+                          bool* needs_copy_engine, Range* cache);
+    bool overlaps_pool(uint64_t a, uint64_t n) const {
+        const uint64_t pend = pool_ + cfg_.pool_bytes;
+        return n && a < pend && pool_ < a + n;
+    }
+
+    // ---- launch building
+    struct Seg {
+        uint64_t user;
+        uint64_t nbytes_flags;
+        const uint32_t* pages;
+        uint32_t n_pages;
+    };
+    template <Mode M>
+    t2i_status launch_segments(const std::vector<Seg>& segs, cudaStream_t stream);
+    template <Mode M, bool GENERAL>
+    t2i_status launch_group(const std::vector<Seg>& segs, cudaStream_t stream);
+    template <Mode M, bool GENERAL, int BLOB>
+    t2i_status launch_one(const std::vector<SegDesc>& sd, const std::vector<uint32_t>& pages, uint32_t n_units,
+                          cudaStream_t stream);
+    void order_after_last(cudaStream_t s) {
+        if (have_last_ && s != last_stream_) {
+            cudaEventRecord(order_ev_, last_stream_);
+            cudaStreamWaitEvent(s, order_ev_, 0);
+        }
+        last_stream_ = s;
+        have_last_ = true;
+    }
+
+    uint64_t pool_;
+    t2i_store_config cfg_;
+    int device_;
+    Control ctl_;
+    t2i_ctl handle_{};
+    uint32_t page_shift_ = 0, unit_shift_ = 0;
+    int max_ctas_[3][2] = {{1, 1}, {1, 1}, {1, 1}};  // [mode][any alignment]: resident CTAs on the device
+    std::vector<Seg> aligned_, general_;
+    cudaEvent_t order_ev_ = nullptr;
+    cudaStream_t last_stream_ = nullptr;
+    bool have_last_ = false;
+    std::string err_;
+    std::vector<const Object*> objs_;
+    std::vector<Seg> segs_;
+    std::vector<SegDesc> sd_;
+    std::vector<uint32_t> lp_;
+    alignas(16) unsigned char param_buf_[sizeof(LaunchParams<kBlobLarge>)];
+};
+
+t2i_status Store::check_user(const void* p, uint64_t n, bool want_write, bool is_host_flag, uint64_t* dev_addr,
+                             bool* needs_copy_engine, Range* cache) {
+    const uint64_t a = reinterpret_cast<uint64_t>(p);
+    *needs_copy_engine = false;
+    *dev_addr = a;
+    if (n == 0) return T2I_OK;
+    if (!p) {
+        err_ = "null buffer";
+        return T2I_ERR_INVALID;
+    }
+    if (a + n < a) {
+        err_ = "buffer range wraps around";
+        return T2I_ERR_INVALID;
+    }
+    if (overlaps_pool(a, n)) {
+        err_ = "a user buffer overlaps the store's pool";
+        return T2I_ERR_INVALID;
+    }
+    if (!cfg_.check_pointers) {
+        *needs_copy_engine = is_host_flag && cfg_.h2d_mode == 1;
+        return T2I_OK;
+    }
+    if (!(cache->kind != MemKind::Unknown && a >= cache->start && a + n <= cache->end)) {
+        if (!query_range(p, cache)) {
+            err_ = "the CUDA driver cannot describe a buffer pointer";
+            return T2I_ERR_INVALID;
+        }
+    }
+    const Range& r = *cache;
+    switch (r.kind) {
+        case MemKind::Device:
+            if (is_host_flag) {
+                err_ = "src_is_host = 1 but the buffer is device memory";
+                return T2I_ERR_INVALID;
+            }
+            if (r.device != device_) {
+                err_ = "a buffer lives on another device";
+                return T2I_ERR_INVALID;
+            }
+            break;
+        case MemKind::Managed:
+            break;
+        case MemKind::Host:
+            if (!is_host_flag && !want_write) {
+                err_ = "host memory passed as a device source (set src_is_host)";
+                return T2I_ERR_INVALID;
+            }
+            *dev_addr = r.dev_base + (a - r.start);
+            *needs_copy_engine = !want_write && cfg_.h2d_mode == 1;
+            break;
+        case MemKind::Unknown:
+            // pageable host memory: only a host source, through the copy engine
+            if (is_host_flag && !want_write) {
+                *needs_copy_engine = true;
+                return T2I_OK;
+            }
+            err_ = want_write ? "a get destination must be device memory or pinned host memory"
+                              : "unknown source pointer (not device memory; set src_is_host for host memory)";
+            return T2I_ERR_INVALID;
+    }
+    if (a + n > r.end) {
+        err_ = "a buffer range runs past the end of its allocation";
+        return T2I_ERR_INVALID;
+    }
+    return T2I_OK;
+}
+
+template <Mode M, bool GENERAL, int BLOB>
+t2i_status Store::launch_one(const std::vector<SegDesc>& sd, const std::vector<uint32_t>& pages, uint32_t n_units,
+                             cudaStream_t stream) {
+    auto* p = reinterpret_cast<LaunchParams<BLOB>*>(param_buf_);
+    p->h.pool = pool_;
+    p->h.n_seg = static_cast<uint32_t>(sd.size());
+    p->h.n_units = n_units;
+    p->h.page_shift = page_shift_;
+    p->h.unit_shift = unit_shift_;
+    p->h.pages_offset = static_cast<uint32_t>(sd.size() * sizeof(SegDesc));
+    p->h.pad = 0;
+    std::memcpy(p->blob, sd.data(), sd.size() * sizeof(SegDesc));
+    std::memcpy(p->blob + p->h.pages_offset, pages.data(), pages.size() * sizeof(uint32_t));
+    const unsigned grid =
+        static_cast<unsigned>(std::min<uint64_t>(n_units, uint64_t(max_ctas_[int(M)][GENERAL ? 1 : 0])));
+    void* args[] = {p};
+    const void* fn = M == Mode::Put   ? reinterpret_cast<const void*>(scatter_put_kernel<BLOB, GENERAL>)
+                     : M == Mode::Get ? reinterpret_cast<const void*>(gather_get_kernel<BLOB, GENERAL>)
+                                      : reinterpret_cast<const void*>(compact_move_kernel<BLOB>);
+    cudaError_t e = cudaLaunchKernel(fn, dim3(grid), dim3(kThreads), args, 0, stream);
+    if (e != cudaSuccess) {
+        err_ = std::string("kernel launch failed: ") + cudaGetErrorString(e);
+        return T2I_ERR_CUDA;
+    }
+    ctl_.counters().launches++;
+    return T2I_OK;
+}
+
+// Segments whose user address is 16-byte aligned go to the aligned kernels,
+// the others (rare: views at odd offsets) to the any-alignment kernels.
+template <Mode M>
+t2i_status Store::launch_segments(const std::vector<Seg>& segs, cudaStream_t stream) {
+    aligned_.clear();
+    general_.clear();
+    for (const Seg& s : segs) ((s.user & 15u) == 0 ? aligned_ : general_).push_back(s);
+    t2i_status st = T2I_OK;
+    if (!aligned_.empty()) st = launch_group<M, false>(aligned_, stream);
+    if (st == T2I_OK && !general_.empty()) {
+        if (M == Mode::Move) return T2I_ERR_INVALID;  // pool pages are always aligned
+        st = launch_group<(M == Mode::Move ? Mode::Put : M), true>(general_, stream);
+    }
+    return st;
+}
+
+// Packs segments into launches: descriptors and page numbers of as many
+// segments as fit one launch's parameter space; an object whose page list
+// alone does not fit is split at page boundaries.
+template <Mode M, bool GENERAL>
+t2i_status Store::launch_group(const std::vector<Seg>& segs, cudaStream_t stream) {
+    sd_.clear();
+    lp_.clear();
+    uint64_t units = 0;
+    auto flush = [&]() -> t2i_status {
+        if (sd_.empty()) return T2I_OK;
+        const size_t bytes = sd_.size() * sizeof(SegDesc) + lp_.size() * sizeof(uint32_t);
+        t2i_status st;
+        if (bytes <= size_t(kBlobSmall))
+            st = launch_one<M, GENERAL, kBlobSmall>(sd_, lp_, uint32_t(units), stream);
+        else if (bytes <= size_t(kBlobMid))
+            st = launch_one<M, GENERAL, kBlobMid>(sd_, lp_, uint32_t(units), stream);
+        else
+            st = launch_one<M, GENERAL, kBlobLarge>(sd_, lp_, uint32_t(units), stream);
+        sd_.clear();
+        lp_.clear();
+        units = 0;
+        return st;
+    };
+    const uint64_t P = uint64_t(1) << page_shift_;
+    const uint64_t max_pages_per_seg = (kBlobLarge - sizeof(SegDesc)) / sizeof(uint32_t);
+    const uint64_t units_per_page = uint64_t(1) << (page_shift_ - unit_shift_);
+    for (const Seg& s : segs) {
+        const uint64_t nbytes = s.nbytes_flags & ~kCastFlag;
+        const uint64_t flags = s.nbytes_flags & kCastFlag;
+        for (uint64_t p0 = 0; p0 < s.n_pages; p0 += max_pages_per_seg) {
+            const uint64_t np = std::min<uint64_t>(max_pages_per_seg, s.n_pages - p0);
+            const uint64_t off = p0 * P;
+            const uint64_t seg_bytes = std::min<uint64_t>(nbytes - off, np * P);
+            const uint64_t seg_units = (seg_bytes + (uint64_t(1) << unit_shift_) - 1) >> unit_shift_;
+            const size_t need = (sd_.size() + 1) * sizeof(SegDesc) + (lp_.size() + np) * sizeof(uint32_t);
+            if (need > size_t(kBlobLarge) || units + seg_units > 0xFFFFFFFFull - units_per_page) {
+                t2i_status st = flush();
+                if (st != T2I_OK) return st;
+            }
+            SegDesc d;
+            // a get with the cast writes half as many bytes as it reads
+            d.user = s.user + (flags ? off / 2 : off);
+            d.nbytes_flags = seg_bytes | flags;
+            d.unit_begin = static_cast<uint32_t>(units);
+            d.page_begin = static_cast<uint32_t>(lp_.size());
+            sd_.push_back(d);
+            lp_.insert(lp_.end(), s.pages + p0, s.pages + p0 + np);
+            units += seg_units;
+        }
+    }
+    return flush();
+}
+
+t2i_status Store::put(const t2i_put_desc* descs, uint32_t n, t2i_id* ids, cudaStream_t stream) {
+    if (n == 0) return T2I_OK;
+    if (!descs || !ids) {
+        err_ = "put: null descriptor or id array";
+        return T2I_ERR_INVALID;
+    }
+    // 1. check every source before touching the directory
+    std::vector<uint64_t> dev_src(n);
+    std::vector<uint8_t> use_ce(n);
+    Range cache;
+    for (uint32_t i = 0; i < n; ++i) {
+        const t2i_put_desc& d = descs[i];
+        if (d.src_is_host > 1 || d.evictable > 1) {
+            err_ = "put: src_is_host and evictable must be 0 or 1";
+            return T2I_ERR_INVALID;
+        }
+        bool ce = false;
+        if (d.src) {
+            t2i_status st = check_user(d.src, d.nbytes, false, d.src_is_host != 0, &dev_src[i], &ce, &cache);
+            if (st != T2I_OK) {
+                err_ = "put: item " + std::to_string(i) + ": " + err_;
+                return st;
+            }
+        }
+        use_ce[i] = ce;
+    }
+    // 2. plan and commit pages (evicting if needed)
+    t2i_status st = ctl_.put(descs, n, ids, &objs_);
+    if (st != T2I_OK) {
+        err_ = ctl_.error();
+        return st;
+    }
+    // 3. copies, stream-ordered after this store's previous work
+    DeviceGuard g(device_);
+    order_after_last(stream);
+    segs_.clear();
+    const uint64_t P = uint64_t(1) << page_shift_;
+    for (uint32_t i = 0; i < n; ++i) {
+        const Object* o = objs_[i];
+        if (!descs[i].src || o->nbytes == 0) continue;
+        if (use_ce[i]) {
+            // one copy per run of consecutive pages
+            const char* src = static_cast<const char*>(descs[i].src);
+            size_t j = 0;
+            while (j < o->pages.size()) {
+                size_t k = j + 1;
+                while (k < o->pages.size() && o->pages[k] == o->pages[k - 1] + 1) ++k;
+                const uint64_t off = j * P;
+                const uint64_t bytes = std::min<uint64_t>(o->nbytes - off, (k - j) * P);
+                cudaError_t e = cudaMemcpyAsync(reinterpret_cast<void*>(pool_ + uint64_t(o->pages[j]) * P), src + off,
+                                                bytes, cudaMemcpyHostToDevice, stream);
+                if (e != cudaSuccess) {
+                    err_ = std::string("put: host copy failed: ") + cudaGetErrorString(e);
+                    ctl_.rollback_put(ids, n);
+                    return T2I_ERR_CUDA;
+                }
+                ctl_.counters().h2d_copies++;
+                j = k;
+            }
+        } else {
+            segs_.push_back({dev_src[i], o->nbytes, o->pages.data(), uint32_t(o->pages.size())});
+        }
+    }
+    if (!segs_.empty()) {
+        st = launch_segments<Mode::Put>(segs_, stream);
+        if (st != T2I_OK) {
+            ctl_.rollback_put(ids, n);
+            return st;
+        }
+    }
+    return T2I_OK;
+}
+
+t2i_status Store::get(const t2i_get_desc* descs, uint32_t n, t2i_status* per_item, cudaStream_t stream) {
+    if (n == 0) return T2I_OK;
+    if (!descs) {
+        err_ = "get: null descriptor array";
+        return T2I_ERR_INVALID;
+    }
+    // 1. directory (ids, evictions, cast rules) without touching the LRU
+    std::vector<t2i_status> per(n, T2I_OK);
+    std::vector<uint64_t> dev_dst(n, 0);
+    t2i_status first = T2I_OK;
+    uint32_t first_i = 0;
+    Range cache;
+    for (uint32_t i = 0; i < n; ++i) {
+        const t2i_get_desc& d = descs[i];
+        t2i_status s = T2I_OK;
+        const Object* o = ctl_.find(d.id);
+        if (d.cast > 1 || d.reserved != 0) {
+            s = T2I_ERR_INVALID;
+        } else if (!o) {
+            s = ctl_.is_evicted(d.id) ? T2I_ERR_EVICTED : T2I_ERR_NOT_FOUND;
+        } else {
+            const uint64_t out_bytes = d.cast ? o->nbytes / 2 : o->nbytes;
+            if ((d.cast && (o->nbytes % 4 != 0 || (reinterpret_cast<uint64_t>(d.dst) & 1))) ||
+                d.dst_bytes < out_bytes) {
+                s = T2I_ERR_INVALID;
+            } else {
+                bool ce = false;
+                if (check_user(d.dst, out_bytes, true, false, &dev_dst[i], &ce, &cache) != T2I_OK) s = T2I_ERR_INVALID;
+            }
+        }
+        per[i] = s;
+        if (s != T2I_OK && first == T2I_OK) {
+            first = s;
+            first_i = i;
+        }
+    }
+    if (first != T2I_OK) {
+        // nothing is written and the LRU is not touched; misses still count
+        std::string why = err_;
+        for (t2i_status s : per) ctl_.counters().misses += s == T2I_ERR_EVICTED;
+        if (per_item) std::copy(per.begin(), per.end(), per_item);
+        static const char* what[] = {"ok", "invalid", "no space", "id not found", "id was evicted", "cuda"};
+        err_ = "get: item " + std::to_string(first_i) + ": " + what[first] +
+               (first == T2I_ERR_INVALID && !why.empty() ? " (" + why + ")" : "");
+        return first;
+    }
+    // 2. LRU stamps
+    t2i_status st = ctl_.get(descs, n, per_item, &objs_);
+    if (st != T2I_OK) {
+        err_ = ctl_.error();
+        return st;
+    }
+    // 3. one gather launch for the batch (copies and casts together)
+    DeviceGuard g(device_);
+    order_after_last(stream);
+    segs_.clear();
+    for (uint32_t i = 0; i < n; ++i) {
+        const Object* o = objs_[i];
+        if (o->nbytes == 0) continue;
+        segs_.push_back({dev_dst[i], o->nbytes | (descs[i].cast ? kCastFlag : 0), o->pages.data(),
+                         uint32_t(o->pages.size())});
+    }
+    if (segs_.empty()) return T2I_OK;
+    return launch_segments<Mode::Get>(segs_, stream);
+}
+
+t2i_status Store::compact(uint64_t limit_bytes, cudaStream_t stream, uint64_t* moved) {
+    std::vector<t2i_move> moves;
+    t2i_status st = ctl_.compact(limit_bytes, &moves);
+    if (moved) *moved = moves.size();
+    if (st != T2I_OK) {
+        err_ = ctl_.error();
+        return st;
+    }
+    if (moves.empty()) return T2I_OK;
+    DeviceGuard g(device_);
+    order_after_last(stream);
+    segs_.clear();
+    const uint64_t P = uint64_t(1) << page_shift_;
+    // each move is a one-page segment whose source is the old page
+    for (const t2i_move& m : moves)
+        segs_.push_back({pool_ + uint64_t(m.src_page) * P, m.valid_bytes, &m.dst_page, 1u});
+    return launch_segments<Mode::Move>(segs_, stream);
+}
+
+}  // namespace t2i
+
+// ======================================================================= C ABI
+using t2i::Store;
+
+struct t2i_store {
+    Store* s;
+};
+
+extern "C" {
+
+t2i_status t2i_store_create(void* pool_dev, const t2i_store_config* cfg, int device, t2i_store** out) {
+    if (!out) {
+        t2i::set_thread_error("t2i_store_create: null out");
+        return T2I_ERR_INVALID;
+    }
+    *out = nullptr;
+    if (!cfg || !pool_dev) {
+        t2i::set_thread_error("t2i_store_create: null pool or config");
+        return T2I_ERR_INVALID;
+    }
+    const int shift = t2i::log2_exact(cfg->page_bytes);
+    if (shift < 8 || shift > 30) {
+        t2i::set_thread_error("t2i_store_create: page_bytes must be a power of two in [256 B, 1 GiB]");
+        return T2I_ERR_INVALID;
+    }
+    if (cfg->pool_bytes / cfg->page_bytes > 0xFFFFFFFFull || cfg->h2d_mode > 1 || cfg->check_pointers > 1) {
+        t2i::set_thread_error("t2i_store_create: too many pages or a bad flag");
+        return T2I_ERR_INVALID;
+    }
+    if (reinterpret_cast<uint64_t>(pool_dev) & 255) {
+        t2i::set_thread_error("t2i_store_create: the pool must be 256-byte aligned");
+        return T2I_ERR_INVALID;
+    }
+    int ndev = 0;
+    if (cudaGetDeviceCount(&ndev) != cudaSuccess || device < 0 || device >= ndev) {
+        cudaGetLastError();
+        t2i::set_thread_error("t2i_store_create: no such CUDA device");
+        return T2I_ERR_CUDA;
+    }
+    t2i::Range r;
+    if (!t2i::query_range(pool_dev, &r) || r.kind != t2i::MemKind::Device || r.device != device ||
+        reinterpret_cast<uint64_t>(pool_dev) + cfg->pool_bytes > r.end) {
+        t2i::set_thread_error("t2i_store_create: the pool must be device memory of `device` covering pool_bytes");
+        return T2I_ERR_INVALID;
+    }
+    Store* s = nullptr;
+    try {
+        s = new Store(pool_dev, *cfg, device);
+    } catch (const std::bad_alloc&) {
+        t2i::set_thread_error("t2i_store_create: host memory allocation failed");
+        return T2I_ERR_INVALID;
+    }
+    std::string err;
+    t2i_status st = s->init(&err);
+    if (st != T2I_OK) {
+        delete s;
+        t2i::set_thread_error("t2i_store_create: " + err);
+        return st;
+    }
+    *out = new t2i_store{s};
+    return T2I_OK;
+}
+
+t2i_status t2i_store_destroy(t2i_store* store) {
+    if (!store) return T2I_OK;
+    delete store->s;
+    delete store;
+    return T2I_OK;
+}
+
+#define T2I_STORE_CALL(store, expr)                                   \
+    do {                                                              \
+        if (!(store)) return T2I_ERR_INVALID;                         \
+        std::lock_guard<std::mutex> lock((store)->s->mu);             \
+        try {                                                         \
+            return (expr);                                            \
+        } catch (const std::bad_alloc&) {                             \
+            return T2I_ERR_INVALID;                                   \
+        }                                                             \
+    } while (0)
+
+t2i_status t2i_put_batch(t2i_store* store, const t2i_put_desc* descs, uint32_t n, t2i_id* out_ids,
+                         void* cuda_stream) {
+    T2I_STORE_CALL(store, store->s->put(descs, n, out_ids, static_cast<cudaStream_t>(cuda_stream)));
+}
+
+t2i_status t2i_get_batch(t2i_store* store, const t2i_get_desc* descs, uint32_t n, t2i_status* per_item,
+                         void* cuda_stream) {
+    T2I_STORE_CALL(store, store->s->get(descs, n, per_item, static_cast<cudaStream_t>(cuda_stream)));
+}
+
+t2i_status t2i_free(t2i_store* store, const t2i_id* ids, uint32_t n) {
+    T2I_STORE_CALL(store, store->s->free(ids, n));
+}
+
+t2i_status t2i_compact(t2i_store* store, uint64_t limit_bytes, void* cuda_stream, uint64_t* pages_moved) {
+    T2I_STORE_CALL(store, store->s->compact(limit_bytes, static_cast<cudaStream_t>(cuda_stream), pages_moved));
+}
+
+t2i_status t2i_store_stats(const t2i_store* store, t2i_stats* out) {
+    if (!store || !out) return T2I_ERR_INVALID;
+    std::lock_guard<std::mutex> lock(store->s->mu);
+    store->s->ctl().stats(out);
+    return T2I_OK;
+}
+
+const t2i_ctl* t2i_store_ctl(const t2i_store* store) { return store ? store->s->ctl_handle() : nullptr; }
+
+const char* t2i_last_error(const t2i_store* store) {
+    if (!store) return t2i::thread_error();
+    return store->s->error().c_str();
+}
+
+}  // extern "C"

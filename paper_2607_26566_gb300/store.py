@@ -1,0 +1,249 @@
+"""Python binding of the paged tensor store: argument marshalling only.
+
+Every call goes straight to the C ABI of libt2istore.so (include/t2istore.h)
+with the same name; every byte is moved by the library's CUDA kernels (or,
+for host sources on request, the copy engine). Descriptor batches are numpy
+structured arrays with the C layout, so large batches cost one array build,
+not a Python loop per object.
+"""
+from __future__ import annotations
+
+import ctypes as C
+
+import numpy as np
+
+from . import _lib as L
+
+PUT_DTYPE = np.dtype([("src", "<u8"), ("nbytes", "<u8"), ("src_is_host", "<u4"), ("dtype_tag", "<u4"),
+                      ("group", "<u8"), ("order", "<u4"), ("evictable", "<u4")])
+GET_DTYPE = np.dtype([("id", "<u8"), ("dst", "<u8"), ("dst_bytes", "<u8"), ("cast", "<u4"), ("reserved", "<u4")])
+MOVE_DTYPE = np.dtype([("src_page", "<u4"), ("dst_page", "<u4"), ("valid_bytes", "<u8")])
+assert PUT_DTYPE.itemsize == C.sizeof(L.PutDesc) and GET_DTYPE.itemsize == C.sizeof(L.GetDesc)
+assert MOVE_DTYPE.itemsize == C.sizeof(L.Move)
+
+
+class T2IError(RuntimeError):
+    def __init__(self, status: int, message: str):
+        super().__init__(f"{L.STATUS_NAMES.get(status, status)}: {message}")
+        self.status = status
+
+
+def _ptr(x) -> int:
+    """Address of a tensor / array / int."""
+    if x is None:
+        return 0
+    if isinstance(x, int):
+        return x
+    if hasattr(x, "data_ptr"):
+        return int(x.data_ptr())
+    if isinstance(x, np.ndarray):
+        return int(x.ctypes.data)
+    raise TypeError(f"cannot take the address of {type(x)}")
+
+
+def _nbytes(x) -> int:
+    if hasattr(x, "untyped_storage") and hasattr(x, "element_size"):
+        return int(x.numel() * x.element_size())
+    return int(x.nbytes)
+
+
+def _stream(stream) -> int:
+    if stream is None:
+        import torch
+        return int(torch.cuda.current_stream().cuda_stream)
+    if isinstance(stream, int):
+        return stream
+    return int(stream.cuda_stream)
+
+
+def put_descs(srcs, nbytes=None, src_is_host=0, dtype_tag=0, group=0, order=0, evictable=0) -> np.ndarray:
+    """A put descriptor array. ``srcs``: tensors / arrays / addresses (0 or
+    None reserves pages); scalars broadcast."""
+    n = len(srcs)
+    d = np.zeros(n, PUT_DTYPE)
+    d["src"] = [_ptr(s) for s in srcs]
+    d["nbytes"] = [_nbytes(s) for s in srcs] if nbytes is None else nbytes
+    d["src_is_host"] = src_is_host
+    d["dtype_tag"] = dtype_tag
+    d["group"] = group
+    d["order"] = order
+    d["evictable"] = evictable
+    return d
+
+
+def get_descs(ids, dsts=None, dst_bytes=None, cast=0) -> np.ndarray:
+    """A get descriptor array; ``dsts``: tensors / arrays / addresses."""
+    n = len(ids)
+    d = np.zeros(n, GET_DTYPE)
+    d["id"] = ids
+    if dsts is not None:
+        d["dst"] = [_ptr(x) for x in dsts]
+        d["dst_bytes"] = [_nbytes(x) for x in dsts] if dst_bytes is None else dst_bytes
+    elif dst_bytes is not None:
+        d["dst_bytes"] = dst_bytes
+    d["cast"] = cast
+    return d
+
+
+def _as(arr: np.ndarray, ctype, dtype):
+    if arr.dtype != dtype or not arr.flags.c_contiguous:
+        raise TypeError("descriptor array has the wrong layout")
+    return arr.ctypes.data_as(C.POINTER(ctype))
+
+
+class Ctl:
+    """The host control core alone (t2i_ctl_*): page allocator, directory,
+    LRU and compaction planner without device memory."""
+
+    def __init__(self, total_pages: int = 0, page_bytes: int = 0, _borrowed=None, _owner=None):
+        self._lib = L.load()
+        self._owner = _owner
+        if _borrowed is not None:
+            self._h = C.c_void_p(_borrowed)
+            self._owned = False
+            return
+        h = C.c_void_p()
+        st = self._lib.t2i_ctl_create(total_pages, page_bytes, C.byref(h))
+        if st != L.OK:
+            raise T2IError(st, self._lib.t2i_ctl_last_error(None).decode())
+        self._h = h
+        self._owned = True
+
+    def close(self):
+        if getattr(self, "_owned", False) and self._h:
+            self._lib.t2i_ctl_destroy(self._h)
+            self._h = C.c_void_p()
+
+    __del__ = close
+
+    def last_error(self) -> str:
+        return self._lib.t2i_ctl_last_error(self._h).decode()
+
+    def put(self, descs: np.ndarray):
+        ids = np.zeros(len(descs), np.uint64)
+        st = self._lib.t2i_ctl_put(self._h, _as(descs, L.PutDesc, PUT_DTYPE), len(descs),
+                                   ids.ctypes.data_as(C.POINTER(C.c_uint64)))
+        return st, ids
+
+    def get(self, descs: np.ndarray):
+        per = np.zeros(len(descs), np.int32)
+        st = self._lib.t2i_ctl_get(self._h, _as(descs, L.GetDesc, GET_DTYPE), len(descs),
+                                   per.ctypes.data_as(C.POINTER(C.c_int32)))
+        return st, per
+
+    def free(self, ids) -> int:
+        ids = np.ascontiguousarray(ids, np.uint64)
+        return self._lib.t2i_ctl_free(self._h, ids.ctypes.data_as(C.POINTER(C.c_uint64)), len(ids))
+
+    def compact(self, limit_bytes: int, cap: int | None = None):
+        n = C.c_uint64(0)
+        if cap is None:
+            cap = 1 << 16
+        moves = np.zeros(cap, MOVE_DTYPE)
+        st = self._lib.t2i_ctl_compact(self._h, limit_bytes, _as(moves, L.Move, MOVE_DTYPE), cap, C.byref(n))
+        if st == L.ERR_INVALID and n.value > cap:
+            return self.compact(limit_bytes, cap=int(n.value))
+        return st, moves[:n.value].copy() if st == L.OK else moves[:0]
+
+    def object(self, oid: int):
+        """(status, info dict, page list)."""
+        info = L.ObjectInfo()
+        st = self._lib.t2i_ctl_object(self._h, oid, C.byref(info), None, 0)
+        if st != L.OK:
+            return st, None, None
+        pages = np.zeros(max(1, info.n_pages), np.uint32)
+        self._lib.t2i_ctl_object(self._h, oid, C.byref(info), pages.ctypes.data_as(C.POINTER(C.c_uint32)),
+                                 info.n_pages)
+        d = {n: int(getattr(info, n)) for n, _ in L.ObjectInfo._fields_}
+        return st, d, pages[:info.n_pages].tolist()
+
+    def free_pages(self) -> list:
+        n = C.c_uint64(0)
+        self._lib.t2i_ctl_free_pages(self._h, None, 0, C.byref(n))
+        out = np.zeros(max(1, n.value), np.uint32)
+        self._lib.t2i_ctl_free_pages(self._h, out.ctypes.data_as(C.POINTER(C.c_uint32)), n.value, C.byref(n))
+        return out[:n.value].tolist()
+
+    def last_evictions(self) -> list:
+        n = C.c_uint64(0)
+        self._lib.t2i_ctl_last_evictions(self._h, None, 0, C.byref(n))
+        out = np.zeros(max(1, n.value), np.uint64)
+        self._lib.t2i_ctl_last_evictions(self._h, out.ctypes.data_as(C.POINTER(C.c_uint64)), n.value, C.byref(n))
+        return [int(x) for x in out[:n.value]]
+
+    def stats(self) -> dict:
+        s = L.Stats()
+        st = self._lib.t2i_ctl_stats(self._h, C.byref(s))
+        if st != L.OK:
+            raise T2IError(st, "stats")
+        return s.as_dict()
+
+
+class Store:
+    """A store over a device pool (``t2i_store_create``). ``pool`` is a CUDA
+    tensor (kept alive by the store object) or an address with ``pool_bytes``."""
+
+    def __init__(self, pool, page_bytes: int, pool_bytes: int | None = None, device: int | None = None,
+                 h2d_mode: int = 0, check_pointers: int = 1):
+        self._lib = L.load()
+        self.pool = pool
+        if pool_bytes is None:
+            pool_bytes = _nbytes(pool)
+        if device is None:
+            device = int(pool.device.index) if hasattr(pool, "device") else 0
+        self.device = device
+        self.page_bytes = int(page_bytes)
+        self.pool_bytes = int(pool_bytes)
+        cfg = L.StoreConfig(pool_bytes, page_bytes, h2d_mode, check_pointers)
+        h = C.c_void_p()
+        st = self._lib.t2i_store_create(C.c_void_p(_ptr(pool)), C.byref(cfg), device, C.byref(h))
+        if st != L.OK:
+            raise T2IError(st, self._lib.t2i_last_error(None).decode())
+        self._h = h
+        self.ctl = Ctl(_borrowed=self._lib.t2i_store_ctl(h), _owner=self)
+
+    def close(self):
+        if getattr(self, "_h", None):
+            self._lib.t2i_store_destroy(self._h)
+            self._h = None
+
+    __del__ = close
+
+    def last_error(self) -> str:
+        return self._lib.t2i_last_error(self._h).decode()
+
+    def put_batch(self, descs: np.ndarray, stream=None):
+        """(status, ids) -- t2i_put_batch."""
+        ids = np.zeros(len(descs), np.uint64)
+        st = self._lib.t2i_put_batch(self._h, _as(descs, L.PutDesc, PUT_DTYPE), len(descs),
+                                     ids.ctypes.data_as(C.POINTER(C.c_uint64)), _stream(stream))
+        return st, ids
+
+    def get_batch(self, descs: np.ndarray, stream=None, per_item: bool = True):
+        """(status, per-item statuses) -- t2i_get_batch."""
+        per = np.zeros(len(descs), np.int32) if per_item else None
+        st = self._lib.t2i_get_batch(self._h, _as(descs, L.GetDesc, GET_DTYPE), len(descs),
+                                     per.ctypes.data_as(C.POINTER(C.c_int32)) if per_item else None,
+                                     _stream(stream))
+        return st, per
+
+    def free(self, ids) -> int:
+        ids = np.ascontiguousarray(ids, np.uint64)
+        return self._lib.t2i_free(self._h, ids.ctypes.data_as(C.POINTER(C.c_uint64)), len(ids))
+
+    def compact(self, limit_bytes: int, stream=None):
+        """(status, pages moved) -- t2i_compact."""
+        n = C.c_uint64(0)
+        st = self._lib.t2i_compact(self._h, limit_bytes, _stream(stream), C.byref(n))
+        return st, int(n.value)
+
+    def stats(self) -> dict:
+        s = L.Stats()
+        st = self._lib.t2i_store_stats(self._h, C.byref(s))
+        if st != L.OK:
+            raise T2IError(st, "stats")
+        return s.as_dict()
+
+    def check(self, st: int):
+        if st != L.OK:
+            raise T2IError(st, self.last_error())

@@ -1,0 +1,76 @@
+"""The C-ABI library loads and exports every call include/t2istore.h declares,
+with the struct layouts the header gives (CPU only: no compute calls)."""
+import ctypes as C
+import os
+import re
+import subprocess
+
+import pytest
+
+from paper_2607_26566_gb300 import _lib as L
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADERS = [os.path.join(ROOT, "include", f) for f in sorted(os.listdir(os.path.join(ROOT, "include"))) if f.endswith(".h")]
+
+
+def declared_functions():
+    names = []
+    for h in HEADERS:
+        text = open(h).read()
+        text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+        names += re.findall(r"^\s*(?:const\s+)?[A-Za-z_][A-Za-z0-9_ ]*?\**\s*\**(t2i_[a-z0-9_]+)\s*\(", text, flags=re.M)
+    return sorted(set(names))
+
+
+def test_header_declares_the_store_calls():
+    names = declared_functions()
+    for required in ("t2i_store_create", "t2i_put_batch", "t2i_get_batch", "t2i_free", "t2i_compact"):
+        assert required in names
+
+
+def test_every_declared_symbol_is_exported(lib):
+    names = declared_functions()
+    assert names
+    for n in names:
+        assert hasattr(lib, n), n
+    assert set(names) == set(L.PROTOTYPES), "binding prototypes and header disagree"
+
+
+def test_only_t2i_symbols_are_exported(lib):
+    out = subprocess.run(["nm", "-D", "--defined-only", L.LIB_PATH], capture_output=True, text=True).stdout
+    syms = [line.split()[-1] for line in out.splitlines() if line.strip()]
+    assert syms and all(s.startswith("t2i_") for s in syms), [s for s in syms if not s.startswith("t2i_")][:5]
+
+
+def test_struct_layouts_match_the_header(tmp_path):
+    prog = tmp_path / "sizes.c"
+    prog.write_text("""
+#include <stdio.h>
+#include <stddef.h>
+#include "t2istore.h"
+int main(void) {
+  printf("%zu %zu %zu %zu %zu %zu\\n", sizeof(t2i_store_config), sizeof(t2i_put_desc), sizeof(t2i_get_desc),
+         sizeof(t2i_move), sizeof(t2i_stats), sizeof(t2i_object_info));
+  printf("%zu %zu %zu\\n", offsetof(t2i_put_desc, group), offsetof(t2i_get_desc, cast), offsetof(t2i_move, valid_bytes));
+  return 0;
+}
+""")
+    exe = tmp_path / "sizes"
+    subprocess.run(["gcc", "-std=c99", "-Wall", "-Werror", "-I" + os.path.join(ROOT, "include"), str(prog), "-o", str(exe)],
+                   check=True)
+    out = subprocess.run([str(exe)], capture_output=True, text=True, check=True).stdout.split()
+    got = [int(x) for x in out]
+    want = [C.sizeof(L.StoreConfig), C.sizeof(L.PutDesc), C.sizeof(L.GetDesc), C.sizeof(L.Move), C.sizeof(L.Stats),
+            C.sizeof(L.ObjectInfo), L.PutDesc.group.offset, L.GetDesc.cast.offset, L.Move.valid_bytes.offset]
+    assert got == want
+
+
+def test_store_create_without_a_gpu_fails_cleanly(lib):
+    import torch
+    if torch.cuda.is_available():
+        pytest.skip("a GPU is present")
+    cfg = L.StoreConfig(1 << 20, 1 << 16, 0, 1)
+    h = C.c_void_p()
+    st = lib.t2i_store_create(C.c_void_p(1 << 20), C.byref(cfg), 0, C.byref(h))
+    assert st in (L.ERR_CUDA, L.ERR_INVALID) and not h.value
+    assert lib.t2i_last_error(None)

@@ -1,0 +1,362 @@
+"""GPU parity: the CUDA store against the oracle, bit for bit (marked gpu).
+
+Small cases compare every byte of every get with the oracle (the definitional
+map plus the oracle's RNE) and the page lists with the oracle's paged model;
+they span several 16 KiB units per page, ragged tails, zero-byte objects,
+misaligned user pointers, pinned-host sources and destinations, evictions and
+compactions.
+"""
+import numpy as np
+import pytest
+import torch
+
+import workloads as W
+from oracle import OracleStore, PutItem
+from oracle.cast import cast_bytes_f32_to_bf16, f32_bits_to_bf16_bits
+from paper_2607_26566_gb300 import Store, get_descs, put_descs
+
+pytestmark = pytest.mark.gpu
+
+DEV = "cuda:0"
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _built(lib):
+    assert torch.cuda.is_available(), "GPU tests need a CUDA device"
+    yield
+
+
+def dev_bytes(a: np.ndarray, offset: int = 0) -> torch.Tensor:
+    """A device uint8 view of ``a`` starting ``offset`` bytes into a fresh allocation."""
+    a = np.ascontiguousarray(a).view(np.uint8).reshape(-1)
+    buf = torch.empty(a.size + offset + 16, dtype=torch.uint8, device=DEV)
+    v = buf[offset:offset + a.size]
+    v.copy_(torch.from_numpy(a))
+    return v
+
+
+def dev_empty(n: int, offset: int = 0) -> torch.Tensor:
+    buf = torch.full((n + offset + 16,), 0xA5, dtype=torch.uint8, device=DEV)
+    return buf[offset:offset + n]
+
+
+def host(t: torch.Tensor) -> np.ndarray:
+    return t.cpu().numpy()
+
+
+def make_store(pool_bytes, page_bytes, **kw):
+    pool = torch.empty(pool_bytes, dtype=torch.uint8, device=DEV)
+    return Store(pool, page_bytes, **kw)
+
+
+def compare_meta(st: Store, ora: OracleStore):
+    assert st.ctl.free_pages() == ora.free_stack
+    for oid, o in ora.objects.items():
+        assert st.ctl.object(oid)[2] == o.pages
+
+
+def check_all_gets(st: Store, ora: OracleStore, rng, with_cast=True):
+    """Get every live object (random alignment, random cast where allowed)
+    and compare with the oracle's get."""
+    ids = [oid for oid, o in ora.objects.items() if o.data is not None]
+    if not ids:
+        return
+    casts = [int(with_cast and ora.objects[i].nbytes % 4 == 0 and rng.random() < 0.3) for i in ids]
+    offs = [int(rng.integers(0, 16)) if rng.random() < 0.3 else 0 for _ in ids]
+    offs = [o & ~1 if c else o for o, c in zip(offs, casts)]
+    dsts = [dev_empty(ora.objects[i].nbytes // (2 if c else 1), o) for i, c, o in zip(ids, casts, offs)]
+    s, per = st.get_batch(get_descs(ids, dsts, cast=casts))
+    assert s == 0, st.last_error()
+    ost, _, outs = ora.get_batch(ids, casts)
+    assert ost == 0
+    torch.cuda.synchronize()
+    for i, d, want in zip(ids, dsts, outs):
+        assert np.array_equal(host(d), want), f"object {i}"
+
+
+def test_tiny_config_bit_exact():
+    """64 MiB pool, 64 KiB pages: put 32, get all, free every third, put 8 more, get all."""
+    C = W.TINY
+    first, more = W.tiny_objects(0)
+    st = make_store(C["pool_bytes"], C["page_bytes"])
+    ora = OracleStore(C["pool_bytes"], C["page_bytes"])
+    srcs = [dev_bytes(x) for x in first]
+    s, ids = st.put_batch(put_descs(srcs))
+    assert s == 0, st.last_error()
+    ost, oids = ora.put_batch([PutItem(x.size, x) for x in first])
+    assert list(ids) == oids
+    rng = np.random.default_rng(0)
+    check_all_gets(st, ora, rng, with_cast=False)
+    gone = [oids[i] for i in W.tiny_freed_indices()]
+    assert st.free(gone) == 0 and ora.free(gone) == 0
+    srcs2 = [dev_bytes(x) for x in more]
+    s, ids2 = st.put_batch(put_descs(srcs2))
+    assert s == 0
+    ora.put_batch([PutItem(x.size, x) for x in more])
+    compare_meta(st, ora)
+    check_all_gets(st, ora, rng, with_cast=False)
+    assert st.stats()["live_objects"] == 30
+
+
+@pytest.mark.parametrize("seed,P,pages", [(0, 256, 64), (1, 4096, 48), (2, 64 * 1024, 24), (3, 2 * 1024 * 1024, 6),
+                                          (4, 32 * 1024, 40), (5, 1024, 200)])
+def test_random_ops_vs_oracle(seed, P, pages):
+    rng = np.random.default_rng(seed)
+    st = make_store(pages * P, P)
+    ora = OracleStore(pages * P, P)
+    keep = []
+    for step in range(60):
+        r = rng.random()
+        if r < 0.45:
+            k = int(rng.integers(1, 6))
+            items, descs_src = [], []
+            for _ in range(k):
+                n = int(rng.integers(0, 3 * P + 1)) if rng.random() < 0.8 else int(rng.integers(0, 64))
+                n -= n % 4 if rng.random() < 0.5 else 0
+                data = rng.integers(0, 256, n, dtype=np.uint8)
+                off = int(rng.integers(0, 16)) if rng.random() < 0.3 else 0
+                t = dev_bytes(data, off)
+                keep.append(t)
+                items.append(PutItem(n, data, group=int(rng.integers(0, 3)), order=int(rng.integers(0, 5)),
+                                     evictable=bool(rng.random() < 0.5)))
+                descs_src.append(t)
+            d = put_descs(descs_src, group=[it.group for it in items], order=[it.order for it in items],
+                          evictable=[int(it.evictable) for it in items])
+            s, ids = st.put_batch(d)
+            ost, oids = ora.put_batch(items)
+            assert s == ost, st.last_error()
+            if s == 0:
+                assert list(ids) == oids
+                assert st.ctl.last_evictions() == ora.last_evictions
+        elif r < 0.65:
+            check_all_gets(st, ora, rng)
+        elif r < 0.85 and ora.objects:
+            ids = [int(x) for x in rng.choice(list(ora.objects), size=min(2, len(ora.objects)), replace=False)]
+            assert st.free(ids) == ora.free(ids) == 0
+        else:
+            limit = int(rng.integers(0, pages + 1)) * P
+            s, moved = st.compact(limit)
+            ost, moves = ora.compact(limit)
+            assert s == ost
+            if s == 0:
+                assert moved == len(moves)
+        compare_meta(st, ora)
+    check_all_gets(st, ora, rng)
+    torch.cuda.synchronize()
+
+
+def test_cast_structured_patterns():
+    """Every rounding case of every exponent through the fused cast."""
+    from tests.test_oracle_cast import structured_patterns
+
+    u = structured_patterns(7).astype(np.uint32)
+    st = make_store(64 << 20, 2 << 20)
+    src = dev_bytes(u.view(np.uint8))
+    s, (i,) = st.put_batch(put_descs([src]))
+    assert s == 0
+    out = torch.empty(u.size, dtype=torch.int16, device=DEV)
+    s, _ = st.get_batch(get_descs([int(i)], [out], cast=1))
+    assert s == 0, st.last_error()
+    got = host(out).view(np.uint16)
+    assert np.array_equal(got, f32_bits_to_bf16_bits(u))
+
+
+def test_cast_exhaustive_2_32():
+    """All 2^32 fp32 bit patterns, in chunks of 2^28, against the oracle's RNE."""
+    chunk = 1 << 28
+    st = make_store(2 << 30, 2 << 20)
+    out = torch.empty(chunk, dtype=torch.int16, device=DEV)
+    base = torch.arange(chunk, dtype=torch.int64, device=DEV)
+    for c in range((1 << 32) // chunk):
+        pat = base + c * chunk                      # the fp32 bit patterns of this chunk
+        bits = torch.where(pat >= 2**31, pat - 2**32, pat).to(torch.int32)
+        s, (i,) = st.put_batch(put_descs([bits]))
+        assert s == 0
+        s, _ = st.get_batch(get_descs([int(i)], [out], cast=1))
+        assert s == 0
+        got = host(out).view(np.uint16)
+        want = f32_bits_to_bf16_bits(np.arange(c * chunk, (c + 1) * chunk, dtype=np.uint64).astype(np.uint32))
+        assert np.array_equal(got, want), f"chunk {c}"
+        assert st.free([int(i)]) == 0
+
+
+def test_handoff_small_vs_oracle():
+    """The handoff workload at reduced tensor sizes, every byte vs the oracle."""
+    specs = W.handoff_specs(2, text_len=40, text_dim=96, pooled_dim=24, lat_c=4, lat_hw=24, img_hw=40)
+    P = 16 * 1024
+    st = make_store(1024 * P, P)
+    ora = OracleStore(1024 * P, P)
+    ci = W.handoff_cast_index()
+    all_ids = []
+    for r in range(12):
+        arrs = W.handoff_request(5, r, specs)
+        srcs = [dev_bytes(a) for a in arrs]
+        s, ids = st.put_batch(put_descs(srcs, dtype_tag=[sp.dtype_tag for sp in specs]))
+        assert s == 0
+        ost, oids = ora.put_batch([PutItem(a.nbytes, a.view(np.uint8).reshape(-1), sp.dtype_tag)
+                                   for a, sp in zip(arrs, specs)])
+        assert list(ids) == oids
+        all_ids.append(oids)
+    compare_meta(st, ora)
+    for oids in all_ids:
+        casts = [1 if j == ci else 0 for j in range(len(specs))]
+        dsts = [dev_empty(ora.objects[i].nbytes // (2 if c else 1)) for i, c in zip(oids, casts)]
+        s, _ = st.get_batch(get_descs(oids, dsts, cast=casts))
+        assert s == 0
+        _, _, outs = ora.get_batch(oids, casts)
+        for d, w in zip(dsts, outs):
+            assert np.array_equal(host(d), w)
+        assert st.free(oids) == ora.free(oids) == 0
+    assert st.stats()["used_pages"] == 0
+
+
+@pytest.mark.parametrize("B", [1, 4, 8])
+def test_handoff_full_size(B):
+    """8 GiB pool, 2 MiB pages, 64 requests in flight, the launch shape the
+    benchmark times. Every non-cast get must equal its input byte for byte
+    (get(put(x)) == x); the cast latents of 8 sampled requests (all at B = 1)
+    are compared with the oracle's RNE."""
+    C = W.HANDOFF
+    specs = W.handoff_specs(B)
+    st = make_store(C["pool_bytes"], C["page_bytes"])
+    ora = OracleStore(C["pool_bytes"], C["page_bytes"], keep_bytes=False)
+    ci = W.handoff_cast_index()
+    reqs, ids_all = [], []
+    for r in range(C["requests"]):
+        ts = W.handoff_request_torch(0, r, specs, DEV)
+        s, ids = st.put_batch(put_descs(ts, nbytes=[sp.nbytes for sp in specs]))
+        assert s == 0, st.last_error()
+        ost, oids = ora.put_batch([PutItem(sp.nbytes, None) for sp in specs])
+        assert list(ids) == oids
+        reqs.append(ts)
+        ids_all.append(oids)
+    compare_meta(st, ora)
+    sampled = set(range(C["requests"])) if B == 1 else set(range(0, C["requests"], 8))
+    for r, (ts, oids) in enumerate(zip(reqs, ids_all)):
+        outs = [torch.empty_like(t) if j != ci else torch.empty(t.shape, dtype=torch.bfloat16, device=DEV)
+                for j, t in enumerate(ts)]
+        casts = [1 if j == ci else 0 for j in range(len(specs))]
+        s, _ = st.get_batch(get_descs(oids, outs, dst_bytes=[sp.nbytes // (2 if c else 1)
+                                                             for sp, c in zip(specs, casts)], cast=casts))
+        assert s == 0, st.last_error()
+        for j, (t, o) in enumerate(zip(ts, outs)):
+            if j != ci:
+                assert torch.equal(t.view(torch.uint8).reshape(-1), o.view(torch.uint8).reshape(-1)), (r, j)
+        if r in sampled:
+            lat = ts[ci].reshape(-1).view(torch.int32).cpu().numpy().view(np.uint32)
+            got = outs[ci].reshape(-1).view(torch.int16).cpu().numpy().view(np.uint16)
+            assert np.array_equal(got, f32_bits_to_bf16_bits(lat)), r
+    for oids in ids_all:
+        assert st.free(oids) == 0
+    assert st.stats()["used_pages"] == 0
+
+
+@pytest.mark.parametrize("h2d_mode", [0, 1])
+def test_host_sources_and_destinations(h2d_mode):
+    """Puts from pinned and pageable host memory, gets into pinned host memory."""
+    rng = np.random.default_rng(9)
+    P = 64 * 1024
+    st = make_store(256 * P, P, h2d_mode=h2d_mode)
+    ora = OracleStore(256 * P, P)
+    datas = [rng.integers(0, 256, int(n), dtype=np.uint8) for n in (1, 100, P, 3 * P + 17, 5 * P, 12345)]
+    pinned = [torch.from_numpy(d).pin_memory() for d in datas[:4]]
+    pageable = [np.ascontiguousarray(d) for d in datas[4:]]
+    s, ids = st.put_batch(put_descs(pinned + pageable, src_is_host=1))
+    assert s == 0, st.last_error()
+    ora.put_batch([PutItem(d.size, d) for d in datas])
+    outs = [torch.empty(d.size, dtype=torch.uint8).pin_memory() for d in datas]
+    s, _ = st.get_batch(get_descs([int(i) for i in ids], outs))
+    assert s == 0, st.last_error()
+    torch.cuda.synchronize()
+    for o, d in zip(outs, datas):
+        assert np.array_equal(o.numpy(), d)
+    stats = st.stats()
+    assert stats["h2d_copies"] > 0                 # pageable sources always take the copy engine
+    assert stats["launches"] >= (2 if h2d_mode == 0 else 1)
+
+
+def test_streams_are_ordered():
+    """Put on one stream, get on another, free, re-put on a third: the store
+    orders its own work across streams."""
+    P = 2 << 20
+    st = make_store(8 * P, P)
+    s1, s2, s3 = torch.cuda.Stream(), torch.cuda.Stream(), torch.cuda.Stream()
+    a = torch.randint(0, 256, (8 * P,), dtype=torch.uint8, device=DEV)
+    b = torch.randint(0, 256, (8 * P,), dtype=torch.uint8, device=DEV)
+    torch.cuda.synchronize()
+    out = torch.empty_like(a)
+    for _ in range(5):
+        s, (i,) = st.put_batch(put_descs([a]), stream=s1)
+        assert s == 0
+        s, _ = st.get_batch(get_descs([int(i)], [out]), stream=s2)
+        assert s == 0
+        assert st.free([int(i)]) == 0
+        s, (j,) = st.put_batch(put_descs([b]), stream=s3)  # reuses the same pages
+        assert s == 0
+        assert st.free([int(j)]) == 0
+        torch.cuda.synchronize()
+        assert torch.equal(out, a)
+
+
+def test_error_paths_never_reach_the_gpu():
+    P = 64 * 1024
+    st = make_store(16 * P, P)
+    x = torch.zeros(1000, dtype=torch.uint8, device=DEV)
+    s, (i,) = st.put_batch(put_descs([x]))
+    assert s == 0
+    pageable = np.zeros(1000, np.uint8)
+    assert st.put_batch(put_descs([pageable]))[0] == 1                  # host memory as a device source
+    assert st.put_batch(put_descs([x], nbytes=[10**6]))[0] == 1        # runs past the allocation
+    assert st.put_batch(put_descs([12345], nbytes=[10]))[0] == 1       # unknown pointer
+    assert st.put_batch(put_descs([st.pool], nbytes=[100]))[0] == 1    # source inside the pool
+    small = torch.empty(10, dtype=torch.uint8, device=DEV)
+    assert st.get_batch(get_descs([int(i)], [small]))[0] == 1          # destination too small
+    assert st.get_batch(get_descs([int(i)], [st.pool], dst_bytes=[1000]))[0] == 1  # into the pool
+    assert st.get_batch(get_descs([int(i)], [pageable]))[0] == 1       # pageable destination
+    assert st.get_batch(get_descs([999], [x]))[0] == 3
+    assert st.put_batch(put_descs([0], nbytes=[17 * P]))[0] == 2
+    odd = torch.empty(1001, dtype=torch.uint8, device=DEV)
+    assert st.get_batch(get_descs([int(i)], [odd[1:]], cast=1))[0] == 1  # cast into an odd address
+    torch.cuda.synchronize()
+    assert st.stats()["live_objects"] == 1 and st.stats()["used_pages"] == 1
+
+
+def test_compaction_moves_bytes_vs_oracle():
+    """A fragmented store compacted to a smaller limit and grown back: every
+    byte vs the oracle, page lists vs the oracle's paged model."""
+    P = 256 * 1024
+    pages = 512
+    tr = W.compaction_trace(11, pages, P, n_ops=4000, lo=4 * W.KiB, hi=24 * W.MiB)
+    st = make_store(pages * P, P)
+    ora = OracleStore(pages * P, P)
+    ids = {}
+    survivors = set(tr.survivors)
+    keep = []
+    for op in tr.ops:
+        if op[0] == "alloc":
+            k, n = op[1], op[2]
+            if k in survivors:
+                data = W.object_bytes(11, k, n)
+                t = dev_bytes(data)
+                keep.append(t)
+                s, (i,) = st.put_batch(put_descs([t]))
+                _, (oi,) = ora.put_batch([PutItem(n, data)])
+            else:
+                s, (i,) = st.put_batch(put_descs([0], nbytes=[n]))
+                _, (oi,) = ora.put_batch([PutItem(n, None)])
+            assert s == 0 and i == oi
+            ids[k] = oi
+        else:
+            oid = ids.pop(op[1])
+            assert st.free([oid]) == ora.free([oid]) == 0
+    compare_meta(st, ora)
+    limit = (pages // 2 + 16) * P
+    s, moved = st.compact(limit)
+    ost, moves = ora.compact(limit)
+    assert s == ost == 0 and moved == len(moves) > 20
+    compare_meta(st, ora)
+    rng = np.random.default_rng(0)
+    check_all_gets(st, ora, rng)
+    s, moved = st.compact(pages * P)
+    assert s == 0 and moved == 0 and ora.compact(pages * P)[0] == 0
+    compare_meta(st, ora)
