@@ -44,7 +44,7 @@ FALLBACK_HBM_GBS = 6800.0
 def parse():
     p = argparse.ArgumentParser()
     p.add_argument("--gpus", type=int, default=1)
-    p.add_argument("--steps", type=int, default=10)
+    p.add_argument("--steps", type=int, default=50)
     p.add_argument("--warmup", type=int, default=3)
     p.add_argument("--impl", default="native", choices=["native", "reference"])
     p.add_argument("--batch", type=int, default=8, help="B of the handoff workload")
@@ -52,6 +52,8 @@ def parse():
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--no-cpu", action="store_true")
     p.add_argument("--sweep", action="store_true", help="also time B = 1 and B = 4")
+    p.add_argument("--pool-gib", type=float, default=None, help="smaller pool (profiling small cases)")
+    p.add_argument("--cpu-seconds", type=float, default=10.0, help="minimum CPU-baseline sample time")
     return p.parse_args()
 
 
@@ -97,7 +99,7 @@ class Clocks:
     def __enter__(self):
         try:
             self.proc = subprocess.Popen(["nvidia-smi", "-i", str(self.index), "--query-gpu=" + self.FIELDS,
-                                          "--format=csv,noheader,nounits", "-lms", "100"],
+                                          "--format=csv,noheader,nounits", "-lms", "50"],
                                          stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
             self.t = threading.Thread(target=self._read, daemon=True)
             self.t.start()
@@ -143,7 +145,8 @@ class Handoff:
     """The handoff workload bound to one store. Descriptor arrays are built
     once; a step issues raw C-ABI calls only."""
 
-    def __init__(self, B: int, requests: int, device, host_buffers: bool = False, seed: int = 0):
+    def __init__(self, B: int, requests: int, device, host_buffers: bool = False, seed: int = 0,
+                 pool_bytes: int | None = None):
         import torch
 
         from paper_2607_26566_gb300 import Store, get_descs, put_descs
@@ -155,7 +158,7 @@ class Handoff:
         self.n_obj = len(self.specs)
         self.requests = requests
         self.ci = W.handoff_cast_index()
-        self.pool = torch.empty(C_["pool_bytes"], dtype=torch.uint8, device=device)
+        self.pool = torch.empty(pool_bytes or C_["pool_bytes"], dtype=torch.uint8, device=device)
         self.store = Store(self.pool, C_["page_bytes"])
         self.lib = self.store._lib
         self.h = self.store._h
@@ -175,9 +178,14 @@ class Handoff:
                              dtype_tag=[sp.dtype_tag for sp in self.specs]) for ts in self.inputs]
         casts = [1 if j == self.ci else 0 for j in range(self.n_obj)]
         self.gd = [get_descs(np.zeros(self.n_obj, np.uint64), outs, cast=casts) for outs in self.outputs]
-        self.pd_p = [d.ctypes.data for d in self.pd]
-        self.gd_p = [d.ctypes.data for d in self.gd]
-        self.ids_p = [self.ids.ctypes.data + 8 * self.n_obj * r for r in range(requests)]
+        from paper_2607_26566_gb300 import _lib as L
+
+        # typed pointers built once: a step makes raw C-ABI calls only
+        self.pd_p = [d.ctypes.data_as(C.POINTER(L.PutDesc)) for d in self.pd]
+        self.gd_p = [d.ctypes.data_as(C.POINTER(L.GetDesc)) for d in self.gd]
+        self.ids_p = [C.cast(C.c_void_p(self.ids.ctypes.data + 8 * self.n_obj * r), C.POINTER(C.c_uint64))
+                      for r in range(requests)]
+        self.all_ids_p = self.ids.ctypes.data_as(C.POINTER(C.c_uint64))
         payload = sum(sp.nbytes for sp in self.specs)
         lat = self.specs[self.ci].nbytes
         self.put_bytes = 2 * payload * requests
@@ -192,7 +200,7 @@ class Handoff:
         for r in range(self.requests):
             if ev is not None:
                 ev["put"][r][0].record()
-            st = lib.t2i_put_batch(h, C.c_void_p(self.pd_p[r]), n, C.c_void_p(self.ids_p[r]), s)
+            st = lib.t2i_put_batch(h, self.pd_p[r], n, self.ids_p[r], s)
             if ev is not None:
                 ev["put"][r][1].record()
             if st:
@@ -201,12 +209,12 @@ class Handoff:
             self.gd[r]["id"] = self.ids[n * r:n * (r + 1)]
             if ev is not None:
                 ev["get"][r][0].record()
-            st = lib.t2i_get_batch(h, C.c_void_p(self.gd_p[r]), n, None, s)
+            st = lib.t2i_get_batch(h, self.gd_p[r], n, None, s)
             if ev is not None:
                 ev["get"][r][1].record()
             if st:
                 raise RuntimeError("get_batch: " + self.store.last_error())
-        st = lib.t2i_free(h, C.c_void_p(self.ids.ctypes.data), len(self.ids))
+        st = lib.t2i_free(h, self.all_ids_p, len(self.ids))
         if st:
             raise RuntimeError("free: " + self.store.last_error())
 
@@ -288,10 +296,12 @@ class Dist:
 
 
 # ----------------------------------------------------------------------------- CPU (oracle)
-def oracle_sample(B: int, n_requests: int):
-    """The oracle as it stands on the host: put + get (latents cast) of
-    ``n_requests`` handoff requests (inputs of one request reused). Returns
-    (GB/s, seconds, bytes)."""
+def oracle_sample(B: int, n_requests: int, min_seconds: float = 0.0, max_steps: int = 1):
+    """The oracle as it stands on the host: steps of the handoff workload (put
+    all ``n_requests`` requests, get them with the latents cast, free them),
+    repeated until ``min_seconds`` have passed or ``max_steps`` were run. The
+    inputs of one request are reused for all requests (the oracle copies
+    them). Returns (GB/s, seconds, bytes, steps)."""
     from oracle import OracleStore, PutItem
 
     specs = W.handoff_specs(B)
@@ -304,16 +314,21 @@ def oracle_sample(B: int, n_requests: int):
     lat = specs[ci].nbytes
     per_req = 2 * payload + 2 * (payload - lat) + 1.5 * lat
     t = time.perf_counter()
-    ids_all = []
-    for _ in range(n_requests):
-        st, ids = store.put_batch([PutItem(x.size, x, sp.dtype_tag) for x, sp in zip(raw, specs)])
-        ids_all.append(ids)
-    for ids in ids_all:
-        store.get_batch(ids, casts)
-    for ids in ids_all:
-        store.free(ids)
-    dt = time.perf_counter() - t
-    return per_req * n_requests / dt / 1e9, dt, per_req * n_requests
+    steps = 0
+    while True:
+        ids_all = []
+        for _ in range(n_requests):
+            st, ids = store.put_batch([PutItem(x.size, x, sp.dtype_tag) for x, sp in zip(raw, specs)])
+            ids_all.append(ids)
+        for ids in ids_all:
+            store.get_batch(ids, casts)
+        for ids in ids_all:
+            store.free(ids)
+        steps += 1
+        dt = time.perf_counter() - t
+        if steps >= max_steps and dt >= min_seconds:
+            break
+    return per_req * n_requests * steps / dt / 1e9, dt, per_req * n_requests * steps, steps
 
 
 # ----------------------------------------------------------------------------- main
@@ -321,13 +336,13 @@ def run_reference(args, dist_ctx):
     if dist_ctx.rank != 0:
         return
     B = args.batch
-    n_req = 8
+    n_req = 8   # a bounded sample of the 64 requests of one step
     for _ in range(args.warmup):
         oracle_sample(B, 1)
     vals = []
     t0 = time.perf_counter()
     for _ in range(args.steps):
-        v, dt, nb = oracle_sample(B, n_req)
+        v, dt, nb, _ = oracle_sample(B, n_req)
         vals.append((v, dt))
     total_t = sum(dt for _, dt in vals)
     total_b = sum(v * dt for v, dt in vals)
@@ -362,7 +377,8 @@ def main():
     device = torch.device("cuda", dist_ctx.local)
     torch.cuda.set_device(device)
     B = args.batch
-    hw = Handoff(B, args.requests, device)
+    pool_bytes = int(args.pool_gib * (1 << 30)) if args.pool_gib else None
+    hw = Handoff(B, args.requests, device, pool_bytes=pool_bytes)
     ms, launches, kern, clocks = time_handoff(hw, args.steps, args.warmup, dist_ctx, per_kernel=True,
                                               clocks_index=dist_ctx.local)
     hw.verify()
@@ -411,9 +427,10 @@ def main():
 
     cpu = None
     if not args.no_cpu and dist_ctx.rank == 0:
-        v, dt, nb = oracle_sample(B, 16)
+        v, dt, nb, n = oracle_sample(B, args.requests, min_seconds=args.cpu_seconds, max_steps=1)
         cpu = {"value": round(v, 3), "unit": "GB/s", "cores": 1, "kind": "oracle",
-               "sample": f"16 B={B} requests put + get (latents cast) by the numpy oracle, {dt:.1f} s"}
+               "sample": f"{n} full step(s) ({args.requests} B={B} requests put, got with the latents cast, "
+                         f"freed) by the numpy oracle in {dt:.1f} s"}
 
     if dist_ctx.rank == 0:
         line = {

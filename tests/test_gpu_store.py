@@ -306,7 +306,7 @@ def test_error_paths_never_reach_the_gpu():
     assert s == 0
     pageable = np.zeros(1000, np.uint8)
     assert st.put_batch(put_descs([pageable]))[0] == 1                  # host memory as a device source
-    assert st.put_batch(put_descs([x], nbytes=[10**6]))[0] == 1        # runs past the allocation
+    assert st.put_batch(put_descs([x], nbytes=[10**8]))[0] == 1        # runs past the allocation
     assert st.put_batch(put_descs([12345], nbytes=[10]))[0] == 1       # unknown pointer
     assert st.put_batch(put_descs([st.pool], nbytes=[100]))[0] == 1    # source inside the pool
     small = torch.empty(10, dtype=torch.uint8, device=DEV)
