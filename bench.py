@@ -195,25 +195,26 @@ class Handoff:
         self.step_bytes = self.put_bytes + self.get_bytes
 
     def step(self, stream, ev=None):
+        """One step. ``ev`` = three events recorded before the puts, between
+        the puts and the gets, and after the gets: each phase is a run of
+        back-to-back launches of one kernel."""
         lib, h, n = self.lib, self.h, self.n_obj
         s = C.c_void_p(stream)
+        if ev is not None:
+            ev[0].record()
         for r in range(self.requests):
-            if ev is not None:
-                ev["put"][r][0].record()
             st = lib.t2i_put_batch(h, self.pd_p[r], n, self.ids_p[r], s)
-            if ev is not None:
-                ev["put"][r][1].record()
             if st:
                 raise RuntimeError("put_batch: " + self.store.last_error())
+        if ev is not None:
+            ev[1].record()
         for r in range(self.requests):
             self.gd[r]["id"] = self.ids[n * r:n * (r + 1)]
-            if ev is not None:
-                ev["get"][r][0].record()
             st = lib.t2i_get_batch(h, self.gd_p[r], n, None, s)
-            if ev is not None:
-                ev["get"][r][1].record()
             if st:
                 raise RuntimeError("get_batch: " + self.store.last_error())
+        if ev is not None:
+            ev[2].record()
         st = lib.t2i_free(h, self.all_ids_p, len(self.ids))
         if st:
             raise RuntimeError("free: " + self.store.last_error())
@@ -233,11 +234,11 @@ def time_handoff(hw: Handoff, steps: int, warmup: int, dist_ctx, per_kernel: boo
     for _ in range(warmup):
         hw.step(stream.cuda_stream)
     torch.cuda.synchronize(hw.device)
-    ev = None
     if per_kernel:
-        mk = lambda: [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
-                      for _ in range(hw.requests)]
-        evs = [{"put": mk(), "get": mk()} for _ in range(steps)]
+        # per step: the put phase and the get phase, each bracketed by events
+        # (an event between two launches would stop the next one from starting
+        # early, so single launches are not bracketed)
+        evs = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(steps)]
     launches0 = hw.store.stats()["launches"]
     clk = Clocks(clocks_index) if clocks_index is not None else None
     if clk:
@@ -247,10 +248,12 @@ def time_handoff(hw: Handoff, steps: int, warmup: int, dist_ctx, per_kernel: boo
     torch.cuda.synchronize(hw.device)
     t0 = torch.cuda.Event(enable_timing=True)
     t1 = torch.cuda.Event(enable_timing=True)
+    torch.cuda.nvtx.range_push("bench_timed")
     t0.record(stream)
     for k in range(steps):
         hw.step(stream.cuda_stream, evs[k] if per_kernel else None)
     t1.record(stream)
+    torch.cuda.nvtx.range_pop()
     torch.cuda.synchronize(hw.device)
     dist_ctx.barrier()
     if clk:
@@ -259,11 +262,13 @@ def time_handoff(hw: Handoff, steps: int, warmup: int, dist_ctx, per_kernel: boo
     launches = hw.store.stats()["launches"] - launches0
     kern = None
     if per_kernel:
-        put_ms = [a.elapsed_time(b) for e in evs for a, b in e["put"]]
-        get_ms = [a.elapsed_time(b) for e in evs for a, b in e["get"]]
+        # a phase holds hw.requests launches of its kernel
+        put_ms = [e[0].elapsed_time(e[1]) / hw.requests for e in evs]
+        get_ms = [e[1].elapsed_time(e[2]) / hw.requests for e in evs]
         kern = {"put_ms": statistics.mean(put_ms), "get_ms": statistics.mean(get_ms),
                 "put_bytes": hw.put_bytes / hw.requests, "get_bytes": hw.get_bytes / hw.requests,
-                "put_total_ms": sum(put_ms), "get_total_ms": sum(get_ms)}
+                "put_total_ms": statistics.mean(put_ms) * hw.requests * steps,
+                "get_total_ms": statistics.mean(get_ms) * hw.requests * steps}
     return ms, launches, kern, (clk.summary() if clk else None)
 
 
@@ -439,7 +444,7 @@ def main():
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "u8+f32->bf16",
             "data": "synthetic",
             "config": {"workload": f"t2i handoff, B={B}, {args.requests} requests in flight",
-                       "pool_bytes": W.HANDOFF["pool_bytes"], "page_bytes": W.HANDOFF["page_bytes"],
+                       "pool_bytes": pool_bytes or W.HANDOFF["pool_bytes"], "page_bytes": W.HANDOFF["page_bytes"],
                        "bytes_per_step": hw_bytes(B, args.requests), "l2": "inputs > L2 (no flush)",
                        "parallelism": f"replicas x{dist_ctx.world}"},
             "hbm_frac": round(value / dist_ctx.world / peak, 4), "hbm_frac_nominal_8tbs": round(value / dist_ctx.world / 8000.0, 4),

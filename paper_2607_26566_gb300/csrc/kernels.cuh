@@ -1,15 +1,21 @@
 // Device code of the paged tensor store: the batched page-table scatter
 // (put), gather (get), gather with a fused fp32 -> bf16 round-to-nearest-even
-// cast, and live-page moves (compaction). All four are one copy engine over
-// "units": a unit is up to U = 2^unit_shift bytes of one object that lie in
-// one page. A launch carries its descriptors in its own parameter space
-// (up to ~31 KiB): no device scratch memory, no host->device descriptor copy.
+// cast, and live-page moves (compaction). All four are one copy engine. A
+// launch carries its descriptors in its own parameter space (up to ~31 KiB):
+// no device scratch memory and no host->device descriptor copy.
+//
+// Work split: the segments of a launch are laid end to end in a "launch byte
+// space" (each starting on a 32-byte granule) and every CTA takes an equal,
+// contiguous share of it, so all CTAs finish together. A CTA walks its share
+// in pieces of at most U = 16 KiB that lie in one page of one segment,
+// mapping each piece to its page through the segment's page list.
 //
 // HBM-bound by construction (2 bytes of traffic per payload byte, 1.5 for the
-// cast): the design goals are fully coalesced 16-byte accesses, enough bytes
-// in flight per SM (4 independent 16-byte loads per thread before the first
-// store, 6 resident CTAs of 256 threads per SM) and a persistent grid sized
-// from the SM count and the occupancy.
+// cast): fully coalesced 16-byte accesses, enough bytes in flight per SM (4
+// independent 16-byte loads per thread before the first store, 5-6 resident
+// CTAs of 256 threads per SM), a persistent grid sized from the SM count and
+// the occupancy, and programmatic dependent launch so that the next launch's
+// set-up overlaps the end of this one.
 #pragma once
 
 #include <cstdint>
@@ -17,11 +23,13 @@
 namespace t2i {
 
 constexpr int kThreads = 256;     // threads per CTA
-constexpr int kVecPerThread = 4;  // 16-byte vectors per thread per unit
+constexpr int kVecPerThread = 4;  // 16-byte vectors per thread per round of a copy loop
 constexpr int kMinBlocks = 6;     // resident CTAs per SM the register budget must allow
 constexpr int kMinBlocksGet = 5;      // same, gather (its cast path needs a few more registers)
 constexpr int kMinBlocksGeneral = 2;  // same, kernels that handle any alignment
-constexpr uint32_t kUnitShiftMax = 14;  // U = 16 KiB = kThreads * kVecPerThread * 16
+constexpr uint32_t kPieceBytes = kThreads * kVecPerThread * 16;  // U = 16 KiB: one round of the copy loop
+constexpr uint32_t kGranule = 32;  // segment starts and CTA shares fall on 32-byte boundaries
+constexpr uint64_t kMinCtaBytes = 16 * 1024;  // smallest share worth a CTA
 
 // One object segment of a launch. For a put/move the user address is the
 // source; for a get it is the destination. Bit 63 of nbytes_flags asks for
@@ -29,18 +37,18 @@ constexpr uint32_t kUnitShiftMax = 14;  // U = 16 KiB = kThreads * kVecPerThread
 struct SegDesc {
     uint64_t user;
     uint64_t nbytes_flags;
-    uint32_t unit_begin;  // first unit of this segment within the launch
+    uint32_t start;       // first granule of this segment in the launch byte space
     uint32_t page_begin;  // first entry of its pages in the launch's page array
 };
 static_assert(sizeof(SegDesc) == 24, "SegDesc layout");
 constexpr uint64_t kCastFlag = uint64_t(1) << 63;
 
 struct LaunchHeader {
-    uint64_t pool;        // pool base address (device)
+    uint64_t pool;          // pool base address (device)
     uint32_t n_seg;
-    uint32_t n_units;
+    uint32_t n_granules;    // size of the launch byte space in granules
     uint32_t page_shift;
-    uint32_t unit_shift;
+    uint32_t piece_bytes;   // min(U, page size)
     uint32_t pages_offset;  // byte offset of the uint32 page array in blob
     uint32_t pad;
 };
@@ -98,7 +106,7 @@ __device__ __forceinline__ uint4 shift_pick(uint4 lo, uint4 hi, uint32_t r) {
 }
 
 // CTA-wide copy of len <= U bytes. The aligned case (both sides 16-byte
-// aligned: every page, every unit of an aligned tensor) is one round of
+// aligned: every page, every piece of an aligned tensor) is one round of
 // kVecPerThread independent 16-byte loads, then the stores.
 __device__ __forceinline__ void cta_copy_aligned(unsigned char* __restrict__ dst,
                                                  const unsigned char* __restrict__ src, uint32_t len) {
@@ -231,13 +239,13 @@ __device__ __forceinline__ void cta_cast_scalar(unsigned char* __restrict__ dst,
     for (uint32_t i = threadIdx.x; i < nf; i += kThreads) d[i] = (uint16_t)bf16_rne_bits(s[i]);
 }
 
-// Largest segment index whose first unit is <= u (segments are non-empty
-// and ordered by unit_begin). All threads search the same u: uniform loads.
-__device__ __forceinline__ uint32_t find_segment(const SegDesc* segs, uint32_t n, uint32_t u) {
+// Largest segment index whose first granule is <= g (segments are non-empty
+// and ordered by start). All threads search the same g: uniform loads.
+__device__ __forceinline__ uint32_t find_segment(const SegDesc* segs, uint32_t n, uint32_t g) {
     uint32_t lo = 0, hi = n - 1;
     while (lo < hi) {
         const uint32_t mid = (lo + hi + 1) >> 1;
-        if (segs[mid].unit_begin <= u)
+        if (segs[mid].start <= g)
             lo = mid;
         else
             hi = mid - 1;
@@ -245,29 +253,49 @@ __device__ __forceinline__ uint32_t find_segment(const SegDesc* segs, uint32_t n
     return lo;
 }
 
-// The unit loop. GENERAL = false: every user address of the launch is
+// Programmatic dependent launch: wait until the previous grid in the stream
+// has completed and its memory is visible (returns at once when this launch
+// has no such dependency), then let the next launch begin its set-up.
+__device__ __forceinline__ void pdl_wait_then_release() {
+    asm volatile("griddepcontrol.wait;" ::: "memory");
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
+// The piece loop. GENERAL = false: every user address of the launch is
 // 16-byte aligned (the host sorts segments into aligned and other launches),
 // so only the vector paths are compiled in and the register budget stays
 // small enough for kMinBlocks resident CTAs per SM. GENERAL = true adds the
 // shifted copies and the element-wise cast for any alignment.
 template <Mode M, bool GENERAL, int BLOB>
-__device__ __forceinline__ void run_units(const LaunchParams<BLOB>& p) {
+__device__ __forceinline__ void run_share(const LaunchParams<BLOB>& p) {
     const SegDesc* segs = reinterpret_cast<const SegDesc*>(p.blob);
     const uint32_t* pages = reinterpret_cast<const uint32_t*>(p.blob + p.h.pages_offset);
     unsigned char* pool = reinterpret_cast<unsigned char*>(p.h.pool);
-    const uint32_t ushift = p.h.unit_shift;
     const uint32_t pshift = p.h.page_shift;
     const uint64_t pmask = (uint64_t(1) << pshift) - 1;
+    const uint64_t piece = p.h.piece_bytes;
+    // this CTA's share of the launch byte space, in whole granules
+    const uint64_t g0 = uint64_t(p.h.n_granules) * blockIdx.x / gridDim.x;
+    const uint64_t g1 = uint64_t(p.h.n_granules) * (blockIdx.x + 1) / gridDim.x;
+    if (g0 == g1) return;
+    uint64_t pos = g0 * kGranule;
+    const uint64_t end = g1 * kGranule;
+    uint32_t i = find_segment(segs, p.h.n_seg, uint32_t(g0));
 #pragma unroll 1
-    for (uint32_t u = blockIdx.x; u < p.h.n_units; u += gridDim.x) {
-        const uint32_t i = find_segment(segs, p.h.n_seg, u);
+    while (pos < end) {
         const SegDesc s = segs[i];
+        const uint64_t lo = uint64_t(s.start) * kGranule;
         const uint64_t nbytes = s.nbytes_flags & ~kCastFlag;
-        const uint32_t k = u - s.unit_begin;
-        const uint64_t off = uint64_t(k) << ushift;
-        const uint32_t len = (uint32_t)umin64(uint64_t(1) << ushift, nbytes - off);
-        const uint32_t page = pages[s.page_begin + (k >> (pshift - ushift))];
-        unsigned char* paddr = pool + (uint64_t(page) << pshift) + (off & pmask);
+        if (pos >= lo + nbytes) {  // past this segment (its padding): next one
+            if (++i >= p.h.n_seg) break;
+            pos = uint64_t(segs[i].start) * kGranule;  // segments are ordered: this is >= pos
+            continue;
+        }
+        const uint64_t off = pos - lo;  // a multiple of kGranule
+        const uint64_t in_page = off & pmask;
+        const uint32_t len = (uint32_t)umin64(umin64(end - pos, nbytes - off), umin64(piece, pmask + 1 - in_page));
+        const uint32_t page = pages[s.page_begin + (off >> pshift)];
+        unsigned char* paddr = pool + (uint64_t(page) << pshift) + in_page;
         unsigned char* uaddr = reinterpret_cast<unsigned char*>(s.user);
         if (M == Mode::Get) {
             if (s.nbytes_flags & kCastFlag) {
@@ -286,6 +314,7 @@ __device__ __forceinline__ void run_units(const LaunchParams<BLOB>& p) {
             else
                 cta_copy_unaligned(paddr, uaddr + off, len);
         }
+        pos += len;
     }
 }
 
@@ -293,16 +322,19 @@ __device__ __forceinline__ void run_units(const LaunchParams<BLOB>& p) {
 template <int BLOB, bool GENERAL>
 __global__ void __launch_bounds__(kThreads, GENERAL ? kMinBlocksGeneral : kMinBlocks)
     scatter_put_kernel(const __grid_constant__ LaunchParams<BLOB> p) {
-    run_units<Mode::Put, GENERAL, BLOB>(p);
+    pdl_wait_then_release();
+    run_share<Mode::Put, GENERAL, BLOB>(p);
 }
 template <int BLOB, bool GENERAL>
 __global__ void __launch_bounds__(kThreads, GENERAL ? kMinBlocksGeneral : kMinBlocksGet)
     gather_get_kernel(const __grid_constant__ LaunchParams<BLOB> p) {
-    run_units<Mode::Get, GENERAL, BLOB>(p);
+    pdl_wait_then_release();
+    run_share<Mode::Get, GENERAL, BLOB>(p);
 }
 template <int BLOB>
 __global__ void __launch_bounds__(kThreads, kMinBlocks) compact_move_kernel(const __grid_constant__ LaunchParams<BLOB> p) {
-    run_units<Mode::Move, false, BLOB>(p);
+    pdl_wait_then_release();
+    run_share<Mode::Move, false, BLOB>(p);
 }
 
 #endif  // __CUDACC__

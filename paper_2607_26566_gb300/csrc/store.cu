@@ -105,7 +105,6 @@ class Store {
         handle_.core = &ctl_;
         handle_.owned = false;
         page_shift_ = log2_exact(cfg.page_bytes);
-        unit_shift_ = std::min<uint32_t>(page_shift_, kUnitShiftMax);
     }
     ~Store() {
         if (order_ev_) {
@@ -180,7 +179,7 @@ class Store {
     template <Mode M, bool GENERAL>
     t2i_status launch_group(const std::vector<Seg>& segs, cudaStream_t stream);
     template <Mode M, bool GENERAL, int BLOB>
-    t2i_status launch_one(const std::vector<SegDesc>& sd, const std::vector<uint32_t>& pages, uint32_t n_units,
+    t2i_status launch_one(const std::vector<SegDesc>& sd, const std::vector<uint32_t>& pages, uint32_t n_granules,
                           cudaStream_t stream);
     void order_after_last(cudaStream_t s) {
         if (have_last_ && s != last_stream_) {
@@ -196,7 +195,7 @@ class Store {
     int device_;
     Control ctl_;
     t2i_ctl handle_{};
-    uint32_t page_shift_ = 0, unit_shift_ = 0;
+    uint32_t page_shift_ = 0;
     int max_ctas_[3][2] = {{1, 1}, {1, 1}, {1, 1}};  // [mode][any alignment]: resident CTAs on the device
     std::vector<Seg> aligned_, general_;
     cudaEvent_t order_ev_ = nullptr;
@@ -278,25 +277,38 @@ t2i_status Store::check_user(const void* p, uint64_t n, bool want_write, bool is
 }
 
 template <Mode M, bool GENERAL, int BLOB>
-t2i_status Store::launch_one(const std::vector<SegDesc>& sd, const std::vector<uint32_t>& pages, uint32_t n_units,
+t2i_status Store::launch_one(const std::vector<SegDesc>& sd, const std::vector<uint32_t>& pages, uint32_t n_granules,
                              cudaStream_t stream) {
     auto* p = reinterpret_cast<LaunchParams<BLOB>*>(param_buf_);
     p->h.pool = pool_;
     p->h.n_seg = static_cast<uint32_t>(sd.size());
-    p->h.n_units = n_units;
+    p->h.n_granules = n_granules;
     p->h.page_shift = page_shift_;
-    p->h.unit_shift = unit_shift_;
+    p->h.piece_bytes = static_cast<uint32_t>(std::min<uint64_t>(kPieceBytes, uint64_t(1) << page_shift_));
     p->h.pages_offset = static_cast<uint32_t>(sd.size() * sizeof(SegDesc));
     p->h.pad = 0;
     std::memcpy(p->blob, sd.data(), sd.size() * sizeof(SegDesc));
     std::memcpy(p->blob + p->h.pages_offset, pages.data(), pages.size() * sizeof(uint32_t));
-    const unsigned grid =
-        static_cast<unsigned>(std::min<uint64_t>(n_units, uint64_t(max_ctas_[int(M)][GENERAL ? 1 : 0])));
+    // every CTA gets at least kMinCtaBytes of the launch (small batches use a
+    // smaller grid); at most the resident CTAs of the whole device
+    const uint64_t want = (uint64_t(n_granules) * kGranule + kMinCtaBytes - 1) / kMinCtaBytes;
+    const unsigned grid = static_cast<unsigned>(
+        std::max<uint64_t>(1, std::min<uint64_t>(want, uint64_t(max_ctas_[int(M)][GENERAL ? 1 : 0]))));
     void* args[] = {p};
     const void* fn = M == Mode::Put   ? reinterpret_cast<const void*>(scatter_put_kernel<BLOB, GENERAL>)
                      : M == Mode::Get ? reinterpret_cast<const void*>(gather_get_kernel<BLOB, GENERAL>)
                                       : reinterpret_cast<const void*>(compact_move_kernel<BLOB>);
-    cudaError_t e = cudaLaunchKernel(fn, dim3(grid), dim3(kThreads), args, 0, stream);
+    cudaLaunchConfig_t lc = {};
+    lc.gridDim = dim3(grid);
+    lc.blockDim = dim3(kThreads);
+    lc.dynamicSmemBytes = 0;
+    lc.stream = stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    lc.attrs = attr;
+    lc.numAttrs = 1;
+    cudaError_t e = cudaLaunchKernelExC(&lc, fn, args);
     if (e != cudaSuccess) {
         err_ = std::string("kernel launch failed: ") + cudaGetErrorString(e);
         return T2I_ERR_CUDA;
@@ -328,25 +340,24 @@ template <Mode M, bool GENERAL>
 t2i_status Store::launch_group(const std::vector<Seg>& segs, cudaStream_t stream) {
     sd_.clear();
     lp_.clear();
-    uint64_t units = 0;
+    uint64_t gran = 0;  // next free granule of the launch byte space
     auto flush = [&]() -> t2i_status {
         if (sd_.empty()) return T2I_OK;
         const size_t bytes = sd_.size() * sizeof(SegDesc) + lp_.size() * sizeof(uint32_t);
         t2i_status st;
         if (bytes <= size_t(kBlobSmall))
-            st = launch_one<M, GENERAL, kBlobSmall>(sd_, lp_, uint32_t(units), stream);
+            st = launch_one<M, GENERAL, kBlobSmall>(sd_, lp_, uint32_t(gran), stream);
         else if (bytes <= size_t(kBlobMid))
-            st = launch_one<M, GENERAL, kBlobMid>(sd_, lp_, uint32_t(units), stream);
+            st = launch_one<M, GENERAL, kBlobMid>(sd_, lp_, uint32_t(gran), stream);
         else
-            st = launch_one<M, GENERAL, kBlobLarge>(sd_, lp_, uint32_t(units), stream);
+            st = launch_one<M, GENERAL, kBlobLarge>(sd_, lp_, uint32_t(gran), stream);
         sd_.clear();
         lp_.clear();
-        units = 0;
+        gran = 0;
         return st;
     };
     const uint64_t P = uint64_t(1) << page_shift_;
     const uint64_t max_pages_per_seg = (kBlobLarge - sizeof(SegDesc)) / sizeof(uint32_t);
-    const uint64_t units_per_page = uint64_t(1) << (page_shift_ - unit_shift_);
     for (const Seg& s : segs) {
         const uint64_t nbytes = s.nbytes_flags & ~kCastFlag;
         const uint64_t flags = s.nbytes_flags & kCastFlag;
@@ -354,9 +365,9 @@ t2i_status Store::launch_group(const std::vector<Seg>& segs, cudaStream_t stream
             const uint64_t np = std::min<uint64_t>(max_pages_per_seg, s.n_pages - p0);
             const uint64_t off = p0 * P;
             const uint64_t seg_bytes = std::min<uint64_t>(nbytes - off, np * P);
-            const uint64_t seg_units = (seg_bytes + (uint64_t(1) << unit_shift_) - 1) >> unit_shift_;
+            const uint64_t seg_gran = (seg_bytes + kGranule - 1) / kGranule;
             const size_t need = (sd_.size() + 1) * sizeof(SegDesc) + (lp_.size() + np) * sizeof(uint32_t);
-            if (need > size_t(kBlobLarge) || units + seg_units > 0xFFFFFFFFull - units_per_page) {
+            if (need > size_t(kBlobLarge) || gran + seg_gran > 0xFFFFFFFFull) {
                 t2i_status st = flush();
                 if (st != T2I_OK) return st;
             }
@@ -364,11 +375,11 @@ t2i_status Store::launch_group(const std::vector<Seg>& segs, cudaStream_t stream
             // a get with the cast writes half as many bytes as it reads
             d.user = s.user + (flags ? off / 2 : off);
             d.nbytes_flags = seg_bytes | flags;
-            d.unit_begin = static_cast<uint32_t>(units);
+            d.start = static_cast<uint32_t>(gran);
             d.page_begin = static_cast<uint32_t>(lp_.size());
             sd_.push_back(d);
             lp_.insert(lp_.end(), s.pages + p0, s.pages + p0 + np);
-            units += seg_units;
+            gran += seg_gran;
         }
     }
     return flush();
