@@ -54,6 +54,9 @@ def parse():
     p.add_argument("--sweep", action="store_true", help="also time B = 1 and B = 4")
     p.add_argument("--pool-gib", type=float, default=None, help="smaller pool (profiling small cases)")
     p.add_argument("--cpu-seconds", type=float, default=10.0, help="minimum CPU-baseline sample time")
+    p.add_argument("--rows", default="weights,adapters,compaction",
+                   help="other hot-path rows timed in the same run (comma list, or 'none')")
+    p.add_argument("--adapter-calls", type=int, default=10_000)
     return p.parse_args()
 
 
@@ -300,6 +303,371 @@ class Dist:
             self.dist.destroy_process_group()
 
 
+# ----------------------------------------------------------------------------- weights
+class WeightRestore:
+    """Weight-cache restore: the bf16 weights of a 57-block DiT (1,140 tensors,
+    11.84 B parameters, 22.05 GiB) put from pinned host memory, one put_batch
+    per block (layer-wise loading), then got with one get_batch into
+    contiguous per-block buffers (each tensor 256-byte aligned in its block)."""
+
+    def __init__(self, device, seed: int = 0, h2d_mode: int = 0, n_blocks: int | None = None):
+        import torch
+
+        from paper_2607_26566_gb300 import Store, get_descs, put_descs
+
+        C_ = W.WEIGHTS
+        self.torch = torch
+        self.device = device
+        specs = W.dit_weight_specs()
+        layout = W.block_layout(specs)
+        if n_blocks is not None:
+            layout = layout[:n_blocks]
+        self.specs, self.layout = specs, layout
+        self.pool = torch.empty(C_["pool_bytes"], dtype=torch.uint8, device=device)
+        self.store = Store(self.pool, C_["page_bytes"], h2d_mode=h2d_mode)
+        self.host = []      # pinned per-block source buffers
+        self.dst = []       # device per-block destination buffers
+        for total, members in layout:
+            d = torch.empty(total, dtype=torch.uint8, device=device)
+            for i, off in members:
+                v = W.weight_values_torch(seed, i, specs[i], device)
+                d[off:off + specs[i].nbytes].copy_(v.view(torch.uint8))
+            h = torch.empty(total, dtype=torch.uint8).pin_memory()
+            h.copy_(d)
+            d.fill_(0xA5)
+            self.host.append(h)
+            self.dst.append(d)
+        torch.cuda.synchronize(device)
+        self.pd = []
+        all_dst, all_bytes = [], []
+        for b, (total, members) in enumerate(layout):
+            base = self.host[b].data_ptr()
+            self.pd.append(put_descs([base + off for _, off in members], nbytes=[specs[i].nbytes for i, _ in members],
+                                     src_is_host=1, dtype_tag=W.DTYPE_BF16, group=0, order=b, evictable=1))
+            all_dst += [self.dst[b].data_ptr() + off for _, off in members]
+            all_bytes += [specs[i].nbytes for i, _ in members]
+        self.n_tensors = len(all_dst)
+        self.gd = get_descs(np.zeros(self.n_tensors, np.uint64), all_dst, dst_bytes=all_bytes)
+        self.payload = sum(all_bytes)
+        self.ids = None
+
+    def put_all(self):
+        ids = []
+        for d in self.pd:
+            st, i = self.store.put_batch(d)
+            self.store.check(st)
+            ids.append(i)
+        self.ids = np.concatenate(ids)
+        self.gd["id"] = self.ids
+
+    def get_all(self):
+        st, _ = self.store.get_batch(self.gd, per_item=False)
+        self.store.check(st)
+
+    def free_all(self):
+        self.store.check(self.store.free(self.ids))
+        self.ids = None
+
+    def verify(self) -> bool:
+        torch = self.torch
+        return all(torch.equal(h.to(self.device, non_blocking=False), d) for h, d in zip(self.host, self.dst))
+
+    def close(self):
+        self.store.close()
+
+
+def time_weights(device, reps: int = 3, h2d_mode: int = 0):
+    import torch
+
+    wr = WeightRestore(device, h2d_mode=h2d_mode)
+    stream = torch.cuda.current_stream(device)
+    wr.put_all()
+    wr.get_all()
+    wr.free_all()
+    torch.cuda.synchronize(device)
+    e = [torch.cuda.Event(enable_timing=True) for _ in range(3)]
+    put_ms, get_ms = [], []
+    launches0 = wr.store.stats()["launches"]
+    for _ in range(reps):
+        e[0].record(stream)
+        wr.put_all()
+        e[1].record(stream)
+        wr.get_all()
+        e[2].record(stream)
+        torch.cuda.synchronize(device)
+        put_ms.append(e[0].elapsed_time(e[1]))
+        get_ms.append(e[1].elapsed_time(e[2]))
+        wr.free_all()
+    launches = (wr.store.stats()["launches"] - launches0) / reps
+    ok = wr.verify()
+    pm, gm = statistics.median(put_ms), statistics.median(get_ms)
+    out = {"workload": "weight restore: 57-block DiT, 1,140 bf16 tensors, 40 GiB pool, 2 MiB pages",
+           "payload_bytes": int(wr.payload), "h2d_mode": h2d_mode,
+           "h2d_put_ms": round(pm, 3), "h2d_link_gbs": round(wr.payload / (pm * 1e-3) / 1e9, 1),
+           "get_ms": round(gm, 3), "get_gbs": round(2 * wr.payload / (gm * 1e-3) / 1e9, 1),
+           "launches_per_rep": launches, "bit_exact": bool(ok)}
+    wr.close()
+    del wr
+    torch.cuda.empty_cache()
+    return out
+
+
+# ----------------------------------------------------------------------------- adapters
+class Adapters:
+    """Multi-tenant adapter cache: 512 LoRA sets (836 bf16 objects each) behind
+    a 16 GiB pool of 256 KiB pages; each call gets a window of 256 objects of a
+    Zipf(1.1)-popular set. A set that is not resident (never loaded, or a
+    window object evicted) is put again from pinned host memory -- evicting
+    least recently used sets -- and the get is retried."""
+
+    def __init__(self, device, seed: int = 0, n_sets: int = 512, n_calls: int = 10_000,
+                 pool_bytes: int | None = None, window: int = 256):
+        import torch
+
+        from paper_2607_26566_gb300 import Store, get_descs, put_descs
+
+        C_ = W.ADAPTERS
+        self.torch = torch
+        self.device = device
+        self.get_descs, self.put_descs = get_descs, put_descs
+        self.window = window
+        self.ranks = W.lora_ranks(seed, n_sets)
+        self.objs = {r: W.lora_objects(int(r)) for r in set(int(x) for x in self.ranks)}
+        self.sizes = {r: np.array([n for _, n in o], np.int64) for r, o in self.objs.items()}
+        self.blocks = {r: np.array([b for b, _ in o], np.int64) for r, o in self.objs.items()}
+        self.rel = {r: np.concatenate([[0], np.cumsum(v)[:-1]]) for r, v in self.sizes.items()}
+        set_bytes = np.array([self.sizes[int(r)].sum() for r in self.ranks], np.int64)
+        self.bank_bytes = int(set_bytes.max() + (1 << 20))
+        bank = W.lora_bank_torch(seed, self.bank_bytes, device)
+        self.bank = torch.empty(self.bank_bytes, dtype=torch.uint8).pin_memory()
+        self.bank.copy_(bank)
+        self.bank_dev = bank   # kept for verification
+        self.off = W.lora_bank_offsets(seed, set_bytes, self.bank_bytes)
+        self.sets, self.starts = W.adapter_calls(seed, n_calls, n_sets, 836, window, C_["zipf_s"])
+        self.pool = torch.empty(pool_bytes or C_["pool_bytes"], dtype=torch.uint8, device=device)
+        self.store = Store(self.pool, C_["page_bytes"])
+        max_window = max(int(np.sort(v)[::-1][:window].sum()) for v in self.sizes.values())
+        self.dst = torch.empty(max_window, dtype=torch.uint8, device=device)
+        self.ids = {}
+        self.loads = 0
+        self.load_bytes = 0
+        self.got_bytes = 0
+        self.calls_done = 0
+
+    def load(self, s: int):
+        r = int(self.ranks[s])
+        old = self.ids.pop(s, None)
+        if old is not None:
+            self.store.check(self.store.free(old))
+        base = self.bank.data_ptr() + int(self.off[s])
+        d = self.put_descs(base + self.rel[r], nbytes=self.sizes[r], src_is_host=1, dtype_tag=W.DTYPE_BF16,
+                           group=s, order=self.blocks[r], evictable=1)
+        st, ids = self.store.put_batch(d)
+        self.store.check(st)
+        self.ids[s] = ids
+        self.loads += 1
+        self.load_bytes += int(self.sizes[r].sum())
+
+    def descs(self, k: int):
+        s, w = int(self.sets[k]), int(self.starts[k])
+        r = int(self.ranks[s])
+        sz = self.sizes[r][w:w + self.window]
+        dst_rel = np.concatenate([[0], np.cumsum(sz)[:-1]])
+        return s, w, self.get_descs(self.ids[s][w:w + self.window], self.dst.data_ptr() + dst_rel, dst_bytes=sz)
+
+    def call(self, k: int, stream=None):
+        s = int(self.sets[k])
+        if s not in self.ids:
+            self.load(s)
+        s, w, d = self.descs(k)
+        st, _ = self.store.get_batch(d, stream=stream, per_item=False)
+        if st == 4:  # EVICTED: reload the whole set and retry
+            self.load(s)
+            s, w, d = self.descs(k)
+            st, _ = self.store.get_batch(d, stream=stream, per_item=False)
+        self.store.check(st)
+        self.got_bytes += int(d["dst_bytes"].sum())
+        self.calls_done += 1
+        return s, w
+
+    def expected(self, s: int, w: int):
+        """The window's bytes as the oracle's get returns them: the set's
+        objects are the bank window at the set's offset, in object order."""
+        r = int(self.ranks[s])
+        a = int(self.off[s]) + int(self.rel[r][w])
+        n = int(self.sizes[r][w:w + self.window].sum())
+        return self.bank_dev[a:a + n]
+
+    def close(self):
+        self.store.close()
+
+
+def time_adapters(device, n_calls: int = 10_000, check_every: int = 500):
+    import torch
+
+    ad = Adapters(device, n_calls=n_calls)
+    stream = torch.cuda.current_stream(device)
+    torch.cuda.synchronize(device)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    s0 = ad.store.stats()
+    t_wall = time.perf_counter()
+    e0.record(stream)
+    bad = 0
+    for k in range(n_calls):
+        s, w = ad.call(k)
+        if check_every and k % check_every == 0:
+            n = ad.expected(s, w).numel()
+            bad += int(not torch.equal(ad.dst[:n], ad.expected(s, w)))
+    e1.record(stream)
+    torch.cuda.synchronize(device)
+    wall = time.perf_counter() - t_wall
+    ms = e0.elapsed_time(e1)
+    s1 = ad.store.stats()
+    # the hit path alone: the same calls again with every set resident
+    # (no misses are possible once a call's set has just been touched)
+    hits_ms, hit_bytes, hit_calls = 0.0, 0, 0
+    h0, h1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    # a set is whole while its first victim (last object: highest layer,
+    # highest id) is live
+    whole = {s for s, ids in ad.ids.items() if ad.store.ctl.object(int(ids[-1]))[0] == 0}
+    resident = [k for k in range(n_calls) if int(ad.sets[k]) in whole][:2000]
+    ok_desc = [ad.descs(k)[2] for k in resident]
+    for d in ok_desc[:20]:
+        ad.store.check(ad.store.get_batch(d, per_item=False)[0])
+    torch.cuda.synchronize(device)
+    h0.record(stream)
+    t_hit = time.perf_counter()
+    for d in ok_desc:
+        st, _ = ad.store.get_batch(d, per_item=False)
+        if st:
+            break
+        hit_bytes += int(d["dst_bytes"].sum())
+        hit_calls += 1
+    h1.record(stream)
+    torch.cuda.synchronize(device)
+    t_hit = time.perf_counter() - t_hit
+    hits_ms = h0.elapsed_time(h1)
+    out = {"workload": "adapters: 512 LoRA sets (ranks 8-64), 16 GiB pool, 256 KiB pages, Zipf(1.1), 256-object gets",
+           "calls": n_calls, "ms": round(ms, 2), "calls_per_s": round(n_calls / (ms * 1e-3), 1),
+           "wall_calls_per_s": round(n_calls / wall, 1),
+           "set_loads": ad.loads, "load_gib": round(ad.load_bytes / 2**30, 2),
+           "evictions": int(s1["evictions"] - s0["evictions"]), "misses": int(s1["misses"] - s0["misses"]),
+           "all_calls_gbs": round((2 * ad.got_bytes + ad.load_bytes) / (ms * 1e-3) / 1e9, 1),
+           "hit_calls": hit_calls, "hit_gbs": round(2 * hit_bytes / (hits_ms * 1e-3) / 1e9, 1),
+           "hit_calls_per_s": round(hit_calls / (hits_ms * 1e-3), 1),
+           "hit_host_calls_per_s": round(hit_calls / t_hit, 1),
+           "checked_windows_bad": bad}
+    ad.close()
+    del ad
+    torch.cuda.empty_cache()
+    return out
+
+
+# ----------------------------------------------------------------------------- compaction
+class Compaction:
+    """Compaction under reclaim: a 64 GiB pool of 2 MiB pages fragmented by
+    the seeded alloc/free trace to ~50% occupancy (objects that die in the
+    trace are reserve puts; survivors carry bytes from a device bank), then
+    compact(48 GiB) to hand a contiguous 16 GiB tail back."""
+
+    def __init__(self, device, seed: int = 1, pool_bytes: int | None = None, limit_bytes: int | None = None,
+                 n_ops: int | None = None, hi: int | None = None):
+        import torch
+
+        from paper_2607_26566_gb300 import put_descs
+
+        C_ = W.COMPACTION
+        self.torch = torch
+        self.device = device
+        self.put_descs = put_descs
+        self.P = C_["page_bytes"]
+        self.pool_bytes = pool_bytes or C_["pool_bytes"]
+        self.limit = limit_bytes or C_["limit_bytes"]
+        self.trace = W.compaction_trace(seed, self.pool_bytes // self.P, self.P, n_ops or C_["n_ops"], C_["lo"],
+                                        hi or C_["hi"], C_["p_free"], C_["settle_frac"])
+        self.bank_bytes = (hi or C_["hi"]) + (1 << 20)
+        g = torch.Generator(device=device)
+        g.manual_seed(seed * 31 + 5)
+        self.bank = torch.randint(0, 256, (self.bank_bytes,), dtype=torch.uint8, device=device, generator=g)
+        rng = W.rng(seed, 7)
+        self.off = {k: int(rng.integers(0, (self.bank_bytes - self.trace.sizes[k]) // 256 + 1)) * 256
+                    for k in self.trace.survivors}
+        self.pool = torch.empty(self.pool_bytes, dtype=torch.uint8, device=device)
+        self.store = None
+
+    def build(self):
+        from paper_2607_26566_gb300 import Store
+
+        if self.store is not None:
+            self.store.close()
+        self.store = Store(self.pool, self.P)
+        surv = set(self.trace.survivors)
+        ids = {}
+        bank = self.bank.data_ptr()
+        for op in self.trace.ops:
+            if op[0] == "alloc":
+                k, n = op[1], op[2]
+                src = bank + self.off[k] if k in surv else 0
+                st, i = self.store.put_batch(self.put_descs([src], nbytes=[n]))
+                self.store.check(st)
+                ids[k] = int(i[0])
+            else:
+                self.store.check(self.store.free([ids.pop(op[1])]))
+        self.ids = ids
+        self.torch.cuda.synchronize(self.device)
+
+    def verify(self) -> bool:
+        """Every survivor got back and compared with its bank window."""
+        torch = self.torch
+        from paper_2607_26566_gb300 import get_descs
+
+        n_max = max(self.trace.sizes[k] for k in self.ids)
+        buf = torch.empty(n_max, dtype=torch.uint8, device=self.device)
+        for k, i in self.ids.items():
+            n = self.trace.sizes[k]
+            self.store.check(self.store.get_batch(get_descs([i], [buf.data_ptr()], dst_bytes=[n]), per_item=False)[0])
+            if not torch.equal(buf[:n], self.bank[self.off[k]:self.off[k] + n]):
+                return False
+        return True
+
+    def close(self):
+        if self.store is not None:
+            self.store.close()
+
+
+def time_compaction(device, reps: int = 3):
+    import torch
+
+    cp = Compaction(device)
+    stream = torch.cuda.current_stream(device)
+    ms, moved_b, moved_p, launches = [], 0, 0, 0
+    for r in range(reps + 1):
+        cp.build()
+        s0 = cp.store.stats()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        st, moved = cp.store.compact(cp.limit)
+        e1.record(stream)
+        torch.cuda.synchronize(device)
+        cp.store.check(st)
+        s1 = cp.store.stats()
+        if r:  # the first repetition warms up
+            ms.append(e0.elapsed_time(e1))
+        moved_b = s1["bytes_moved"] - s0["bytes_moved"]
+        moved_p = moved
+        launches = s1["launches"] - s0["launches"]
+    ok = cp.verify()
+    m = statistics.median(ms)
+    out = {"workload": "compaction: 64 GiB pool, 2 MiB pages, 100,000-op trace, compact to 48 GiB",
+           "pages_moved": int(moved_p), "bytes_moved": int(moved_b), "launches": int(launches),
+           "ms": round(m, 3), "gbs": round(2 * moved_b / (m * 1e-3) / 1e9, 1),
+           "live_objects": len(cp.ids), "bit_exact": bool(ok)}
+    cp.close()
+    del cp
+    torch.cuda.empty_cache()
+    return out
+
+
 # ----------------------------------------------------------------------------- CPU (oracle)
 def oracle_sample(B: int, n_requests: int, min_seconds: float = 0.0, max_steps: int = 1):
     """The oracle as it stands on the host: steps of the handoff workload (put
@@ -430,6 +798,19 @@ def main():
         del he
         torch.cuda.empty_cache()
 
+    rows = {}
+    wanted = [] if args.rows == "none" else [r.strip() for r in args.rows.split(",") if r.strip()]
+    if "weights" in wanted:
+        rows["weights"] = time_weights(device)
+    if "adapters" in wanted:
+        rows["adapters"] = time_adapters(device, n_calls=args.adapter_calls)
+    if "compaction" in wanted:
+        rows["compaction"] = time_compaction(device)
+    for r in rows.values():
+        for k in ("get_gbs", "gbs", "hit_gbs"):
+            if k in r:
+                r[k.replace("gbs", "hbm_frac")] = round(r[k] / peak, 4)
+
     cpu = None
     if not args.no_cpu and dist_ctx.rank == 0:
         v, dt, nb, n = oracle_sample(B, args.requests, min_seconds=args.cpu_seconds, max_steps=1)
@@ -449,7 +830,7 @@ def main():
                        "parallelism": f"replicas x{dist_ctx.world}"},
             "hbm_frac": round(value / dist_ctx.world / peak, 4), "hbm_frac_nominal_8tbs": round(value / dist_ctx.world / 8000.0, 4),
             "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e, "gpu_launches": int(launches),
-            "clocks": clocks, "sweep": sweep or None,
+            "clocks": clocks, "sweep": sweep or None, "rows": rows or None,
         }
         print(json.dumps(line), flush=True)
     dist_ctx.close()

@@ -56,12 +56,19 @@ def _stream(stream) -> int:
     return int(stream.cuda_stream)
 
 
+def _addrs(xs):
+    if isinstance(xs, np.ndarray) and xs.dtype.kind in "iu":
+        return xs
+    return [_ptr(x) for x in xs]
+
+
 def put_descs(srcs, nbytes=None, src_is_host=0, dtype_tag=0, group=0, order=0, evictable=0) -> np.ndarray:
-    """A put descriptor array. ``srcs``: tensors / arrays / addresses (0 or
-    None reserves pages); scalars broadcast."""
+    """A put descriptor array. ``srcs``: tensors / arrays / addresses (an
+    integer numpy array of addresses is taken as is; 0 or None reserves
+    pages); scalars broadcast."""
     n = len(srcs)
     d = np.zeros(n, PUT_DTYPE)
-    d["src"] = [_ptr(s) for s in srcs]
+    d["src"] = _addrs(srcs)
     d["nbytes"] = [_nbytes(s) for s in srcs] if nbytes is None else nbytes
     d["src_is_host"] = src_is_host
     d["dtype_tag"] = dtype_tag
@@ -77,7 +84,7 @@ def get_descs(ids, dsts=None, dst_bytes=None, cast=0) -> np.ndarray:
     d = np.zeros(n, GET_DTYPE)
     d["id"] = ids
     if dsts is not None:
-        d["dst"] = [_ptr(x) for x in dsts]
+        d["dst"] = _addrs(dsts)
         d["dst_bytes"] = [_nbytes(x) for x in dsts] if dst_bytes is None else dst_bytes
     elif dst_bytes is not None:
         d["dst_bytes"] = dst_bytes
