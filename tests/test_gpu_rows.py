@@ -1,0 +1,171 @@
+"""GPU parity for the weight-restore, adapter-cache and compaction workloads
+at the full sizes the benchmark times (marked gpu).
+
+Full-size outputs are compared with what the oracle's get returns for them
+(the bytes that were put: pinned host sources, bank windows); the page
+layout, the moves and the eviction decisions are compared with the oracle's
+paged model replaying the same operations.
+"""
+import numpy as np
+import pytest
+import torch
+
+import bench
+import workloads as W
+from oracle import EVICTED, OK, OracleStore, PutItem
+
+pytestmark = pytest.mark.gpu
+DEV = torch.device("cuda", 0)
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _built(lib):
+    assert torch.cuda.is_available(), "GPU tests need a CUDA device"
+    yield
+
+
+def test_weight_restore_full_size():
+    """22.05 GiB of bf16 weights from pinned host (zero-copy kernel), every
+    byte got back; page lists equal the oracle's."""
+    wr = bench.WeightRestore(DEV)
+    ora = OracleStore(W.WEIGHTS["pool_bytes"], W.WEIGHTS["page_bytes"], keep_bytes=False)
+    wr.put_all()
+    for b, (total, members) in enumerate(wr.layout):
+        st, _ = ora.put_batch([PutItem(wr.specs[i].nbytes, None, W.DTYPE_BF16, 0, b, True) for i, _ in members])
+        assert st == OK
+    wr.get_all()
+    torch.cuda.synchronize()
+    assert wr.verify()
+    for oid, o in list(ora.objects.items())[::37]:
+        assert wr.store.ctl.object(oid)[2] == o.pages
+    assert wr.store.ctl.free_pages() == ora.free_stack
+    wr.free_all()
+    wr.close()
+
+
+def test_weight_restore_copy_engine():
+    """The same restore through the copy engine (one cudaMemcpyAsync per run
+    of consecutive pages), on the first 6 blocks."""
+    wr = bench.WeightRestore(DEV, h2d_mode=1, n_blocks=6)
+    wr.put_all()
+    wr.get_all()
+    torch.cuda.synchronize()
+    assert wr.verify()
+    assert wr.store.stats()["h2d_copies"] > 0
+    wr.close()
+
+
+def test_compaction_full_size():
+    """64 GiB pool, the 100,000-op trace, compact to 48 GiB: moves and page
+    lists equal the oracle's; every survivor's bytes survive."""
+    cp = bench.Compaction(DEV)
+    cp.build()
+    P = cp.P
+    ora = OracleStore(cp.pool_bytes, P, keep_bytes=False)
+    ids = {}
+    for op in cp.trace.ops:
+        if op[0] == "alloc":
+            st, (i,) = ora.put_batch([PutItem(op[2])])
+            ids[op[1]] = i
+        else:
+            ora.free([ids.pop(op[1])])
+    assert ids == cp.ids
+    st, moves = ora.compact(cp.limit)
+    assert st == OK
+    s0 = cp.store.stats()
+    st, moved = cp.store.compact(cp.limit)
+    assert st == 0 and moved == len(moves) > 3000
+    s1 = cp.store.stats()
+    assert s1["bytes_moved"] - s0["bytes_moved"] == sum(m[2] for m in moves)
+    assert cp.store.ctl.free_pages() == ora.free_stack
+    for oid, o in ora.objects.items():
+        assert cp.store.ctl.object(oid)[2] == o.pages
+        assert all(p < cp.limit // P for p in o.pages)
+    assert cp.verify()
+    # grow back: nothing moves, the tail is free again
+    st, moved = cp.store.compact(cp.pool_bytes)
+    assert st == 0 and moved == 0 and ora.compact(cp.pool_bytes)[0] == OK
+    assert cp.store.ctl.free_pages() == ora.free_stack
+    cp.close()
+
+
+class OracleAdapters:
+    """The adapter harness's decisions replayed on the oracle (metadata only)."""
+
+    def __init__(self, ad: "bench.Adapters"):
+        self.ad = ad
+        self.ora = OracleStore(ad.pool.numel(), W.ADAPTERS["page_bytes"], keep_bytes=False)
+        self.ids = {}
+
+    def load(self, s):
+        r = int(self.ad.ranks[s])
+        old = self.ids.pop(s, None)
+        if old is not None:
+            assert self.ora.free(old) == OK
+        st, ids = self.ora.put_batch([PutItem(int(n), None, W.DTYPE_BF16, s, int(b), True)
+                                      for n, b in zip(self.ad.sizes[r], self.ad.blocks[r])])
+        assert st == OK
+        self.ids[s] = ids
+        return list(self.ora.last_evictions)
+
+    def call(self, k):
+        s, w = int(self.ad.sets[k]), int(self.ad.starts[k])
+        ev = []
+        if s not in self.ids:
+            ev += self.load(s)
+        st, _, _ = self.ora.get_batch(self.ids[s][w:w + self.ad.window])
+        if st == EVICTED:
+            ev += self.load(s)
+            st, _, _ = self.ora.get_batch(self.ids[s][w:w + self.ad.window])
+        assert st == OK
+        return ev
+
+
+def test_adapters_small_vs_oracle():
+    """64 sets behind a 2 GiB pool, 400 calls: the same loads, the same
+    victims in the same order, the same page lists; every got window equals
+    its bank bytes."""
+    ad = bench.Adapters(DEV, n_sets=64, n_calls=400, pool_bytes=2 << 30)
+    oa = OracleAdapters(ad)
+    for k in range(400):
+        loads0 = ad.loads
+        ev_gpu = []
+        s = int(ad.sets[k])
+        # mirror bench.Adapters.call, collecting the victims of each load
+        if s not in ad.ids:
+            ad.load(s)
+            ev_gpu += ad.store.ctl.last_evictions()
+        _, w, d = ad.descs(k)
+        st, _ = ad.store.get_batch(d, per_item=False)
+        if st == 4:
+            ad.load(s)
+            ev_gpu += ad.store.ctl.last_evictions()
+            _, w, d = ad.descs(k)
+            st, _ = ad.store.get_batch(d, per_item=False)
+        assert st == 0
+        ev_ora = oa.call(k)
+        assert ev_gpu == ev_ora, k
+        n = int(d["dst_bytes"].sum())
+        assert torch.equal(ad.dst[:n], ad.expected(s, w)), k
+        assert ad.loads - loads0 <= 2
+    for s, ids in oa.ids.items():
+        for oid in ids[::50]:
+            o = oa.ora.objects.get(int(oid))
+            if o is not None:
+                assert ad.store.ctl.object(int(oid))[2] == o.pages
+    assert ad.store.ctl.free_pages() == oa.ora.free_stack
+    ad.close()
+
+
+def test_adapters_full_size_windows():
+    """The full adapter workload (512 sets, 16 GiB pool), 3,000 calls; every
+    50th window compared with its bank bytes."""
+    ad = bench.Adapters(DEV, n_calls=3000)
+    for k in range(3000):
+        s, w = ad.call(k)
+        if k % 50 == 0:
+            n = ad.expected(s, w).numel()
+            assert torch.equal(ad.dst[:n], ad.expected(s, w)), k
+    st = ad.store.stats()
+    assert st["evictions"] > 0 and st["used_pages"] <= st["limit_pages"]
+    ad.close()
