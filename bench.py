@@ -57,6 +57,9 @@ def parse():
     p.add_argument("--rows", default="weights,adapters,compaction",
                    help="other hot-path rows timed in the same run (comma list, or 'none')")
     p.add_argument("--adapter-calls", type=int, default=10_000)
+    p.add_argument("--rows-only", action="store_true", help="skip the handoff headline (profiling a row)")
+    p.add_argument("--compaction-gib", type=int, default=None,
+                   help="smaller compaction pool (GiB; the limit is 3/4 of it): profiling small cases")
     return p.parse_args()
 
 
@@ -635,10 +638,14 @@ class Compaction:
             self.store.close()
 
 
-def time_compaction(device, reps: int = 3):
+def time_compaction(device, reps: int = 3, pool_gib: int | None = None):
     import torch
 
-    cp = Compaction(device)
+    if pool_gib:
+        cp = Compaction(device, pool_bytes=pool_gib << 30, limit_bytes=(pool_gib << 30) * 3 // 4,
+                        n_ops=max(2000, 100_000 * pool_gib // 64), hi=min(W.COMPACTION["hi"], (pool_gib << 30) // 128))
+    else:
+        cp = Compaction(device)
     stream = torch.cuda.current_stream(device)
     ms, moved_b, moved_p, launches = [], 0, 0, 0
     for r in range(reps + 1):
@@ -658,7 +665,8 @@ def time_compaction(device, reps: int = 3):
         launches = s1["launches"] - s0["launches"]
     ok = cp.verify()
     m = statistics.median(ms)
-    out = {"workload": "compaction: 64 GiB pool, 2 MiB pages, 100,000-op trace, compact to 48 GiB",
+    out = {"workload": ("compaction: 64 GiB pool, 2 MiB pages, 100,000-op trace, compact to 48 GiB" if not pool_gib
+                        else f"compaction (small case): {pool_gib} GiB pool, compact to 3/4"),
            "pages_moved": int(moved_p), "bytes_moved": int(moved_b), "launches": int(launches),
            "ms": round(m, 3), "gbs": round(2 * moved_b / (m * 1e-3) / 1e9, 1),
            "live_objects": len(cp.ids), "bit_exact": bool(ok)}
@@ -735,6 +743,22 @@ def run_reference(args, dist_ctx):
     print(json.dumps(line), flush=True)
 
 
+def run_rows(args, device, peak):
+    rows = {}
+    wanted = [] if args.rows == "none" else [r.strip() for r in args.rows.split(",") if r.strip()]
+    if "weights" in wanted:
+        rows["weights"] = time_weights(device)
+    if "adapters" in wanted:
+        rows["adapters"] = time_adapters(device, n_calls=args.adapter_calls)
+    if "compaction" in wanted:
+        rows["compaction"] = time_compaction(device, pool_gib=args.compaction_gib)
+    for r in rows.values():
+        for k in ("get_gbs", "gbs", "hit_gbs"):
+            if k in r:
+                r[k.replace("gbs", "hbm_frac")] = round(r[k] / peak, 4)
+    return rows
+
+
 def main():
     args = parse()
     dist_ctx = Dist(args.gpus)
@@ -749,6 +773,10 @@ def main():
     b.ensure_built()
     device = torch.device("cuda", dist_ctx.local)
     torch.cuda.set_device(device)
+    if args.rows_only:
+        print(json.dumps({"rows": run_rows(args, device, peaks()[0])}), flush=True)
+        dist_ctx.close()
+        return
     B = args.batch
     pool_bytes = int(args.pool_gib * (1 << 30)) if args.pool_gib else None
     hw = Handoff(B, args.requests, device, pool_bytes=pool_bytes)
@@ -798,18 +826,7 @@ def main():
         del he
         torch.cuda.empty_cache()
 
-    rows = {}
-    wanted = [] if args.rows == "none" else [r.strip() for r in args.rows.split(",") if r.strip()]
-    if "weights" in wanted:
-        rows["weights"] = time_weights(device)
-    if "adapters" in wanted:
-        rows["adapters"] = time_adapters(device, n_calls=args.adapter_calls)
-    if "compaction" in wanted:
-        rows["compaction"] = time_compaction(device)
-    for r in rows.values():
-        for k in ("get_gbs", "gbs", "hit_gbs"):
-            if k in r:
-                r[k.replace("gbs", "hbm_frac")] = round(r[k] / peak, 4)
+    rows = run_rows(args, device, peak)
 
     cpu = None
     if not args.no_cpu and dist_ctx.rank == 0:
