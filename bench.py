@@ -389,7 +389,7 @@ def time_weights(device, reps: int = 3, h2d_mode: int = 0):
     wr.free_all()
     torch.cuda.synchronize(device)
     e = [torch.cuda.Event(enable_timing=True) for _ in range(3)]
-    put_ms, get_ms = [], []
+    put_ms, get_ms, get_kern_ms = [], [], []
     launches0 = wr.store.stats()["launches"]
     for _ in range(reps):
         e[0].record(stream)
@@ -400,14 +400,21 @@ def time_weights(device, reps: int = 3, h2d_mode: int = 0):
         torch.cuda.synchronize(device)
         put_ms.append(e[0].elapsed_time(e[1]))
         get_ms.append(e[1].elapsed_time(e[2]))
+        gate(device)   # the same get behind a gate: its launches alone
+        e[1].record(stream)
+        wr.get_all()
+        e[2].record(stream)
+        torch.cuda.synchronize(device)
+        get_kern_ms.append(e[1].elapsed_time(e[2]))
         wr.free_all()
     launches = (wr.store.stats()["launches"] - launches0) / reps
     ok = wr.verify()
-    pm, gm = statistics.median(put_ms), statistics.median(get_ms)
+    pm, gm, gk = statistics.median(put_ms), statistics.median(get_ms), statistics.median(get_kern_ms)
     out = {"workload": "weight restore: 57-block DiT, 1,140 bf16 tensors, 40 GiB pool, 2 MiB pages",
            "payload_bytes": int(wr.payload), "h2d_mode": h2d_mode,
            "h2d_put_ms": round(pm, 3), "h2d_link_gbs": round(wr.payload / (pm * 1e-3) / 1e9, 1),
-           "get_ms": round(gm, 3), "get_gbs": round(2 * wr.payload / (gm * 1e-3) / 1e9, 1),
+           "get_call_ms": round(gm, 3), "get_call_gbs": round(2 * wr.payload / (gm * 1e-3) / 1e9, 1),
+           "get_kernel_ms": round(gk, 3), "get_gbs": round(2 * wr.payload / (gk * 1e-3) / 1e9, 1),
            "launches_per_rep": launches, "bit_exact": bool(ok)}
     wr.close()
     del wr
@@ -638,7 +645,19 @@ class Compaction:
             self.store.close()
 
 
-def time_compaction(device, reps: int = 3, pool_gib: int | None = None):
+def gate(device, ms: float = 20.0):
+    """Occupy the stream for ``ms`` with torch's bounded sleep kernel, so that
+    the host work of the next call (planning, descriptor packing) happens
+    while the GPU is busy and events after the gate time the kernels alone."""
+    import torch
+
+    torch.cuda._sleep(int(ms * 1e-3 * 2.0e9))
+
+
+def time_compaction(device, reps: int = 2, pool_gib: int | None = None):
+    """Call-level time (events around t2i_compact with an idle GPU, so the
+    host's planning is included) and kernel-level time (the same call behind a
+    gate: the compaction launches alone), each the median of ``reps``."""
     import torch
 
     if pool_gib:
@@ -647,11 +666,15 @@ def time_compaction(device, reps: int = 3, pool_gib: int | None = None):
     else:
         cp = Compaction(device)
     stream = torch.cuda.current_stream(device)
-    ms, moved_b, moved_p, launches = [], 0, 0, 0
-    for r in range(reps + 1):
+    call_ms, kern_ms, moved_b, moved_p, launches = [], [], 0, 0, 0
+    for r in range(2 * reps + 1):
         cp.build()
+        gated = r % 2 == 1
         s0 = cp.store.stats()
         e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        torch.cuda.synchronize(device)
+        if gated:
+            gate(device)
         e0.record(stream)
         st, moved = cp.store.compact(cp.limit)
         e1.record(stream)
@@ -659,16 +682,17 @@ def time_compaction(device, reps: int = 3, pool_gib: int | None = None):
         cp.store.check(st)
         s1 = cp.store.stats()
         if r:  # the first repetition warms up
-            ms.append(e0.elapsed_time(e1))
+            (kern_ms if gated else call_ms).append(e0.elapsed_time(e1))
         moved_b = s1["bytes_moved"] - s0["bytes_moved"]
         moved_p = moved
         launches = s1["launches"] - s0["launches"]
     ok = cp.verify()
-    m = statistics.median(ms)
+    cm, km = statistics.median(call_ms), statistics.median(kern_ms)
     out = {"workload": ("compaction: 64 GiB pool, 2 MiB pages, 100,000-op trace, compact to 48 GiB" if not pool_gib
                         else f"compaction (small case): {pool_gib} GiB pool, compact to 3/4"),
            "pages_moved": int(moved_p), "bytes_moved": int(moved_b), "launches": int(launches),
-           "ms": round(m, 3), "gbs": round(2 * moved_b / (m * 1e-3) / 1e9, 1),
+           "kernel_ms": round(km, 3), "gbs": round(2 * moved_b / (km * 1e-3) / 1e9, 1),
+           "call_ms": round(cm, 3), "call_gbs": round(2 * moved_b / (cm * 1e-3) / 1e9, 1),
            "live_objects": len(cp.ids), "bit_exact": bool(ok)}
     cp.close()
     del cp

@@ -281,21 +281,31 @@ __device__ __forceinline__ void run_share(const LaunchParams<BLOB>& p) {
     uint64_t pos = g0 * kGranule;
     const uint64_t end = g1 * kGranule;
     uint32_t i = find_segment(segs, p.h.n_seg, uint32_t(g0));
+    // the current segment and page stay in registers until the walk leaves them
+    SegDesc s = segs[i];
+    uint64_t lo = uint64_t(s.start) * kGranule;
+    uint64_t nbytes = s.nbytes_flags & ~kCastFlag;
+    uint64_t page_idx = ~uint64_t(0);
+    unsigned char* page_base = nullptr;
 #pragma unroll 1
     while (pos < end) {
-        const SegDesc s = segs[i];
-        const uint64_t lo = uint64_t(s.start) * kGranule;
-        const uint64_t nbytes = s.nbytes_flags & ~kCastFlag;
         if (pos >= lo + nbytes) {  // past this segment (its padding): next one
             if (++i >= p.h.n_seg) break;
-            pos = uint64_t(segs[i].start) * kGranule;  // segments are ordered: this is >= pos
+            s = segs[i];
+            lo = uint64_t(s.start) * kGranule;  // segments are ordered: this is >= pos
+            nbytes = s.nbytes_flags & ~kCastFlag;
+            page_idx = ~uint64_t(0);
+            pos = lo;
             continue;
         }
         const uint64_t off = pos - lo;  // a multiple of kGranule
         const uint64_t in_page = off & pmask;
+        if ((off >> pshift) != page_idx) {
+            page_idx = off >> pshift;
+            page_base = pool + (uint64_t(pages[s.page_begin + page_idx]) << pshift);
+        }
         const uint32_t len = (uint32_t)umin64(umin64(end - pos, nbytes - off), umin64(piece, pmask + 1 - in_page));
-        const uint32_t page = pages[s.page_begin + (off >> pshift)];
-        unsigned char* paddr = pool + (uint64_t(page) << pshift) + in_page;
+        unsigned char* paddr = page_base + in_page;
         unsigned char* uaddr = reinterpret_cast<unsigned char*>(s.user);
         if (M == Mode::Get) {
             if (s.nbytes_flags & kCastFlag) {
