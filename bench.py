@@ -279,31 +279,50 @@ def time_handoff(hw: Handoff, steps: int, warmup: int, dist_ctx, per_kernel: boo
 
 
 class Dist:
-    def __init__(self, n):
+    """Rank bookkeeping for N independent replicas (one store per GPU; the
+    store has no cross-GPU step, so the only collectives are the timing
+    barrier and the max / sum of the ranks' numbers)."""
+
+    def __init__(self, backend: str | None = None, init: bool = True):
         self.world = int(os.environ.get("WORLD_SIZE", "1"))
         self.rank = int(os.environ.get("RANK", "0"))
         self.local = int(os.environ.get("LOCAL_RANK", "0"))
-        self.on = self.world > 1
+        self.on = self.world > 1 and init
+        self.backend = None
         if self.on:
+            import torch
             import torch.distributed as dist
             self.dist = dist
-            dist.init_process_group("nccl" if os.environ.get("T2I_BENCH_GLOO") is None else "gloo")
+            self.backend = backend or ("nccl" if torch.cuda.is_available() else "gloo")
+            dist.init_process_group(self.backend)
 
     def barrier(self):
         if self.on:
             self.dist.barrier()
 
-    def max(self, x: float) -> float:
+    def _reduce(self, x: float, op) -> float:
         if not self.on:
             return x
         import torch
-        t = torch.tensor([x], dtype=torch.float64, device=f"cuda:{self.local}" if torch.cuda.is_available() else "cpu")
-        self.dist.all_reduce(t, op=self.dist.ReduceOp.MAX)
+        dev = f"cuda:{self.local}" if self.backend == "nccl" else "cpu"
+        t = torch.tensor([x], dtype=torch.float64, device=dev)
+        self.dist.all_reduce(t, op=op)
         return float(t.item())
+
+    def max(self, x: float) -> float:
+        return self._reduce(x, self.dist.ReduceOp.MAX if self.on else None)
+
+    def sum(self, x: float) -> float:
+        return self._reduce(x, self.dist.ReduceOp.SUM if self.on else None)
 
     def close(self):
         if self.on:
             self.dist.destroy_process_group()
+
+
+def job_gbs(bytes_per_rank: float, ms_max: float, dist_ctx: "Dist") -> float:
+    """Whole-job GB/s: the bytes every rank moved over the slowest rank's time."""
+    return dist_ctx.sum(bytes_per_rank) / (ms_max * 1e-3) / 1e9
 
 
 # ----------------------------------------------------------------------------- weights
@@ -785,7 +804,8 @@ def run_rows(args, device, peak):
 
 def main():
     args = parse()
-    dist_ctx = Dist(args.gpus)
+    # the reference arm runs on rank 0 alone and needs no process group
+    dist_ctx = Dist(init=args.impl != "reference")
     if args.impl == "reference":
         run_reference(args, dist_ctx)
         dist_ctx.close()
@@ -808,8 +828,7 @@ def main():
                                               clocks_index=dist_ctx.local)
     hw.verify()
     ms_max = dist_ctx.max(ms)
-    total_bytes = hw.step_bytes * args.steps * dist_ctx.world
-    value = total_bytes / (ms_max * 1e-3) / 1e9
+    value = job_gbs(hw.step_bytes * args.steps, ms_max, dist_ctx)
     peak, peak_kind = peaks()
 
     # dominant kernel: the one with more total time in the timed region
@@ -844,7 +863,7 @@ def main():
         e_steps = max(2, min(args.steps, 3))
         ms_e, _, _, _ = time_handoff(he, e_steps, 1, dist_ctx, per_kernel=False)
         ms_e = dist_ctx.max(ms_e)
-        e2e = {"value": round(he.step_bytes * e_steps * dist_ctx.world / (ms_e * 1e-3) / 1e9, 2), "unit": "GB/s",
+        e2e = {"value": round(job_gbs(he.step_bytes * e_steps, ms_e, dist_ctx), 2), "unit": "GB/s",
                "h2d_bytes_per_step": int(he.h2d_bytes), "d2h_bytes_per_step": int(he.d2h_bytes),
                "path": "t2i_put_batch / t2i_get_batch with pinned host sources and destinations"}
         del he

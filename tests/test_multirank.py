@@ -1,0 +1,70 @@
+"""The replica path of the benchmark on CPU: two gloo ranks (world size 2)
+run the same barrier / max / sum bookkeeping the GPU ranks use; the
+reference arm prints only on rank 0."""
+import json
+import os
+import socket
+import subprocess
+import sys
+
+import torch.multiprocessing as mp
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+def _free_port():
+    s = socket.socket()
+    s.bind(("127.0.0.1", 0))
+    port = s.getsockname()[1]
+    s.close()
+    return port
+
+
+def _worker(rank, world, port, q):
+    os.environ.update(RANK=str(rank), WORLD_SIZE=str(world), LOCAL_RANK=str(rank), MASTER_ADDR="127.0.0.1",
+                      MASTER_PORT=str(port))
+    sys.path.insert(0, ROOT)
+    import bench
+
+    d = bench.Dist(backend="gloo")
+    d.barrier()
+    slowest = d.max(10.0 + rank)            # ms of this rank
+    gbs = bench.job_gbs(1e9 * (rank + 1), slowest, d)
+    d.barrier()
+    q.put((rank, slowest, gbs))
+    d.close()
+
+
+def test_two_gloo_ranks():
+    ctx = mp.get_context("spawn")
+    q = ctx.Queue()
+    port = _free_port()
+    procs = [ctx.Process(target=_worker, args=(r, 2, port, q)) for r in range(2)]
+    for p in procs:
+        p.start()
+    out = sorted(q.get(timeout=120) for _ in procs)
+    for p in procs:
+        p.join(timeout=60)
+        assert p.exitcode == 0
+    # both ranks agree: slowest rank 11 ms, 3 GB in total -> 3 GB / 11 ms
+    for rank, slowest, gbs in out:
+        assert slowest == 11.0
+        assert abs(gbs - 3.0 / 0.011) < 1e-6
+
+
+def test_reference_arm_prints_on_rank0_only():
+    env = dict(os.environ, RANK="1", WORLD_SIZE="2", LOCAL_RANK="1")
+    r = subprocess.run([sys.executable, os.path.join(ROOT, "bench.py"), "--impl", "reference", "--steps", "1",
+                        "--warmup", "0"], capture_output=True, text=True, env=env, timeout=300)
+    assert r.returncode == 0 and r.stdout.strip() == ""
+
+
+def test_single_process_dist_is_a_no_op():
+    sys.path.insert(0, ROOT)
+    import bench
+
+    d = bench.Dist()
+    assert not d.on and d.max(3.5) == 3.5 and d.sum(2.0) == 2.0
+    assert abs(bench.job_gbs(2e9, 1000.0, d) - 2.0) < 1e-12
+    line = {"impl": "reference"}
+    assert json.loads(json.dumps(line)) == line
