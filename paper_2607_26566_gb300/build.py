@@ -58,21 +58,26 @@ def is_stale() -> bool:
     return any(os.path.getmtime(f) > t for f in _inputs())
 
 
-def build(verbose: bool = False, ptxas_info: bool = False) -> str:
-    """Compiles and links the library; returns its path. Raises on failure."""
-    os.makedirs(BUILD, exist_ok=True)
+def build(verbose: bool = False, ptxas_info: bool = False, defines=(), out: str | None = None,
+          build_dir: str | None = None) -> str:
+    """Compiles and links the library; returns its path. Raises on failure.
+    ``defines`` (e.g. ["T2I_TUNE_VEC=8"]) and ``out`` build a variant of the
+    kernels' launch shape elsewhere (tuning sweeps)."""
+    lib_path = out or LIB
+    bdir = build_dir or BUILD
+    os.makedirs(bdir, exist_ok=True)
     cuda = _cuda_home()
     nvcc = os.path.join(cuda, "bin", "nvcc")
     inc = ["-I" + INCLUDE, "-I" + CSRC, "-I" + os.path.join(cuda, "include")]
     jobs = []
     for f in CXX_SOURCES:
-        obj = os.path.join(BUILD, f + ".o")
+        obj = os.path.join(bdir, f + ".o")
         jobs.append(([os.environ.get("CXX", "g++"), "-O2", "-std=c++17", "-fPIC", "-Wall", "-c",
                       os.path.join(CSRC, f), "-o", obj] + inc, obj))
     for f in CU_SOURCES:
-        obj = os.path.join(BUILD, f + ".o")
+        obj = os.path.join(bdir, f + ".o")
         cmd = [nvcc, "-O3", "-std=c++17", *ARCH, "-lineinfo", "-Xcompiler", "-fPIC,-Wall",
-               "-c", os.path.join(CSRC, f), "-o", obj] + inc
+               "-c", os.path.join(CSRC, f), "-o", obj] + inc + ["-D" + d for d in defines]
         if ptxas_info:
             cmd += ["-Xptxas", "-v"]
         jobs.append((cmd, obj))
@@ -89,7 +94,7 @@ def build(verbose: bool = False, ptxas_info: bool = False) -> str:
         objs.append(obj)
     if errors:
         raise RuntimeError("compilation failed:\n" + "\n".join(errors))
-    tmp = LIB + ".tmp"
+    tmp = lib_path + ".tmp"
     link = [nvcc, "-shared", *ARCH, "-o", tmp, *objs, "-cudart", "static", "-lpthread",
             "-Xlinker", "--version-script=" + os.path.join(CSRC, "exports.map")]
     r = subprocess.run(link, stdout=subprocess.PIPE, stderr=subprocess.STDOUT, text=True)
@@ -97,8 +102,8 @@ def build(verbose: bool = False, ptxas_info: bool = False) -> str:
         sys.stderr.write(r.stdout)
     if r.returncode:
         raise RuntimeError("link failed: " + " ".join(link))
-    os.replace(tmp, LIB)
-    return LIB
+    os.replace(tmp, lib_path)
+    return lib_path
 
 
 def ensure_built() -> str:

@@ -22,10 +22,26 @@
 
 namespace t2i {
 
-constexpr int kThreads = 256;     // threads per CTA
-constexpr int kVecPerThread = 4;  // 16-byte vectors per thread per round of a copy loop
-constexpr int kMinBlocks = 6;     // resident CTAs per SM the register budget must allow
-constexpr int kMinBlocksGet = 5;      // same, gather (its cast path needs a few more registers)
+// Launch shape (overridable at compile time for tuning sweeps).
+#ifndef T2I_TUNE_THREADS
+#define T2I_TUNE_THREADS 256
+#endif
+#ifndef T2I_TUNE_VEC
+#define T2I_TUNE_VEC 4
+#endif
+#ifndef T2I_TUNE_MIN_BLOCKS
+#define T2I_TUNE_MIN_BLOCKS 6
+#endif
+#ifndef T2I_TUNE_MIN_BLOCKS_GET
+#define T2I_TUNE_MIN_BLOCKS_GET 5
+#endif
+#ifndef T2I_TUNE_CACHE
+#define T2I_TUNE_CACHE 0  // 0: streaming (.cs) loads and stores; 1: default caching; 2: loads bypass L1
+#endif
+constexpr int kThreads = T2I_TUNE_THREADS;          // threads per CTA
+constexpr int kVecPerThread = T2I_TUNE_VEC;         // 16-byte vectors per thread per round of a copy loop
+constexpr int kMinBlocks = T2I_TUNE_MIN_BLOCKS;     // resident CTAs per SM the register budget must allow
+constexpr int kMinBlocksGet = T2I_TUNE_MIN_BLOCKS_GET;  // same, gather (its cast path needs a few more registers)
 constexpr int kMinBlocksGeneral = 2;  // same, kernels that handle any alignment
 constexpr uint32_t kPieceBytes = kThreads * kVecPerThread * 16;  // U = 16 KiB: one round of the copy loop
 constexpr uint32_t kGranule = 32;  // segment starts and CTA shares fall on 32-byte boundaries
@@ -71,8 +87,22 @@ enum class Mode { Put, Get, Move };
 __device__ __forceinline__ uint64_t umin64(uint64_t a, uint64_t b) { return a < b ? a : b; }
 
 // ---------------------------------------------------------------- loads/stores
+#if T2I_TUNE_CACHE == 0
 __device__ __forceinline__ uint4 ld_stream(const uint4* p) { return __ldcs(p); }
 __device__ __forceinline__ void st_stream(uint4* p, const uint4& v) { __stcs(p, v); }
+#elif T2I_TUNE_CACHE == 1
+__device__ __forceinline__ uint4 ld_stream(const uint4* p) { return *p; }
+__device__ __forceinline__ void st_stream(uint4* p, const uint4& v) { *p = v; }
+#else
+__device__ __forceinline__ uint4 ld_stream(const uint4* p) {
+    uint4 v;
+    asm volatile("ld.global.nc.L1::no_allocate.v4.u32 {%0, %1, %2, %3}, [%4];"
+                 : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
+                 : "l"(p));
+    return v;
+}
+__device__ __forceinline__ void st_stream(uint4* p, const uint4& v) { __stcs(p, v); }
+#endif
 
 // fp32 -> bf16, round to nearest even, on bit patterns: add just under half
 // an ulp of bf16, plus one when the kept part is odd, and drop 16 bits (the
