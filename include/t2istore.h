@@ -71,15 +71,19 @@ typedef struct t2i_store_config {
  * evictable, least recently used model first, higher layers first.        */
 typedef struct t2i_put_desc {
     const void* src;      /* nbytes to copy: device memory of the store's device, or host memory
-                             when src_is_host = 1. NULL reserves pages and copies nothing (the
-                             object's bytes are undefined until overwritten by nobody: a
-                             placeholder that only takes capacity).                          */
+                             when src_is_host = 1. NULL reserves pages and copies nothing: the
+                             object takes capacity and its bytes are undefined.              */
     uint64_t nbytes;      /* object size; 0 is allowed (no pages)                            */
     uint32_t src_is_host; /* 1 = src is host memory (pinned or pageable)                      */
     uint32_t dtype_tag;   /* opaque tag kept in the directory                                 */
     uint64_t group;       /* LRU group: one model or one adapter set                          */
     uint32_t order;       /* layer index inside the group; the highest is evicted first        */
     uint32_t evictable;   /* 1 = cached weights (may be evicted); 0 = intermediate (never)      */
+    uint32_t consumers;   /* > 0: the object is freed by the store after this many successful
+                             gets of it (each occurrence in a get batch counts once): an
+                             intermediate reclaimed when no downstream consumer needs it any
+                             more (§5.3). 0 = freed only by t2i_free (or evicted).           */
+    uint32_t reserved;    /* must be 0                                                        */
 } t2i_put_desc;
 
 /* ---- get ------------------------------------------------------------------
@@ -110,6 +114,7 @@ typedef struct t2i_stats {
     uint64_t pages_moved, bytes_moved;
     uint64_t launches;   /* kernels launched by the store                                    */
     uint64_t h2d_copies; /* copy-engine copies issued for host sources                        */
+    uint64_t reclaimed;  /* objects freed by the store after their last declared consumer    */
 } t2i_stats;
 
 typedef struct t2i_object_info {
@@ -119,6 +124,8 @@ typedef struct t2i_object_info {
     uint32_t order;
     uint32_t evictable;
     uint32_t n_pages;
+    uint32_t consumers_left; /* gets still expected before the store frees it (0 = none)   */
+    uint32_t reserved;
 } t2i_object_info;
 
 /* =========================================================================
@@ -153,9 +160,21 @@ t2i_status t2i_put_batch(t2i_store* store, const t2i_put_desc* descs, uint32_t n
  * OK / NOT_FOUND / EVICTED / INVALID per item. If any item fails, the call
  * returns the first failing status in descriptor order and writes nothing.
  * The same id may appear more than once. Objects reserved with src = NULL
- * return whatever their pages hold.                                          */
+ * return whatever their pages hold. Objects put with consumers > 0 count one
+ * consumer per successful item; those that reach zero are freed once the
+ * call's copies are enqueued (stream order keeps their pages intact until
+ * the copies have run).                                                      */
 t2i_status t2i_get_batch(t2i_store* store, const t2i_get_desc* descs, uint32_t n, t2i_status* per_item,
                          void* cuda_stream);
+
+/* As t2i_get_batch, but the copies start only after `wait_event` (a
+ * cudaEvent_t recorded by the producer, e.g. on another stream) has
+ * completed: the consumer issues the fetch where its execution needs the
+ * tensor, and the store orders it after the producer (§5.2, callback-based
+ * fetching). wait_event = NULL behaves as t2i_get_batch. The wait is a
+ * cudaStreamWaitEvent on cuda_stream: the host never blocks.               */
+t2i_status t2i_get_batch_after(t2i_store* store, const t2i_get_desc* descs, uint32_t n, t2i_status* per_item,
+                               void* cuda_stream, void* wait_event);
 
 /* Returns the pages of n objects to the free stack (paper §5.3: data is
  * reclaimed when no consumer needs it). Host-only: stream order makes reuse

@@ -10,7 +10,7 @@ What the store computes, and where the paper fixes it:
   Intermediate tensors are written once and read by their consumers, never
   updated (§5.3, "Backend-as-a-Service Paradigm": immutability), and are
   reclaimed once no consumer needs them (same paragraph) -- here by an explicit
-  ``free``. A producer writes its output into the local store and a consumer
+  ``free`` or after a declared number of consumers (reading 9). A producer writes its output into the local store and a consumer
   later pulls it into its own buffer (§5.2, "Efficient and flexible data
   fetching").
 * Capacity. The paper manages its arena with a buddy allocator (§5.2); the
@@ -54,6 +54,10 @@ Readings where the paper is silent (each also listed in the design doc):
    grows the store back.
 8. A put descriptor without data reserves pages and copies nothing; the
    object's bytes are undefined (the allocation half of a pull, §5.2).
+9. Reclaim by consumer count (§5.3: tensors are reclaimed once no downstream
+   function needs them): an object put with k > 0 consumers is freed after
+   its k-th successful get item; a get frees the objects it brought to zero
+   at its end, in the order of the items that brought them there.
 """
 from __future__ import annotations
 
@@ -79,6 +83,7 @@ class PutItem:
     group: int = 0
     order: int = 0
     evictable: bool = False
+    consumers: int = 0
 
 
 @dataclass
@@ -90,6 +95,7 @@ class _Object:
     evictable: bool
     pages: list = field(default_factory=list)
     data: np.ndarray | None = None
+    consumers_left: int = 0
 
 
 class OracleStore:
@@ -115,7 +121,7 @@ class OracleStore:
         self.group_last: dict[int, int] = {}
         self.last_evictions: list[int] = []
         self.stats = dict(bytes_put=0, bytes_got=0, gets=0, misses=0, evictions=0,
-                          pages_moved=0, bytes_moved=0, puts=0)
+                          pages_moved=0, bytes_moved=0, puts=0, reclaimed=0)
 
     # -- accounting ---------------------------------------------------------
     def used_pages(self) -> int:
@@ -186,7 +192,7 @@ class OracleStore:
             oid = self.next_id
             self.next_id += 1
             self.objects[oid] = _Object(n, int(it.dtype_tag), int(it.group), int(it.order), bool(it.evictable),
-                                        pages, data if self.keep_bytes else None)
+                                        pages, data if self.keep_bytes else None, int(it.consumers))
             self._touch(int(it.group))
             self.stats["bytes_put"] += n
             self.stats["puts"] += 1
@@ -223,6 +229,7 @@ class OracleStore:
         if bad:
             return bad[0], per, []
         outs = []
+        consumed = []
         for oid, c in zip(ids, casts):
             o = self.objects[int(oid)]
             self._touch(o.group)
@@ -232,6 +239,13 @@ class OracleStore:
             outs.append(raw)
             self.stats["bytes_got"] += o.nbytes
             self.stats["gets"] += 1
+            if o.consumers_left > 0:
+                o.consumers_left -= 1
+                if o.consumers_left == 0:
+                    consumed.append(int(oid))
+        for oid in consumed:          # reading 9: no consumer needs them any more
+            self._release(oid)
+            self.stats["reclaimed"] += 1
         return OK, per, outs
 
     # -- free ---------------------------------------------------------------

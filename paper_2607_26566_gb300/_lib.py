@@ -23,7 +23,7 @@ class StoreConfig(C.Structure):
 class PutDesc(C.Structure):
     _fields_ = [("src", C.c_void_p), ("nbytes", C.c_uint64), ("src_is_host", C.c_uint32),
                 ("dtype_tag", C.c_uint32), ("group", C.c_uint64), ("order", C.c_uint32),
-                ("evictable", C.c_uint32)]
+                ("evictable", C.c_uint32), ("consumers", C.c_uint32), ("reserved", C.c_uint32)]
 
 
 class GetDesc(C.Structure):
@@ -39,7 +39,7 @@ class Stats(C.Structure):
     _fields_ = [(n, C.c_uint64) for n in (
         "total_pages", "limit_pages", "used_pages", "free_pages", "live_objects",
         "bytes_put", "bytes_got", "puts", "gets", "misses", "evictions",
-        "pages_moved", "bytes_moved", "launches", "h2d_copies")]
+        "pages_moved", "bytes_moved", "launches", "h2d_copies", "reclaimed")]
 
     def as_dict(self) -> dict:
         return {n: int(getattr(self, n)) for n, _ in self._fields_}
@@ -47,7 +47,8 @@ class Stats(C.Structure):
 
 class ObjectInfo(C.Structure):
     _fields_ = [("nbytes", C.c_uint64), ("group", C.c_uint64), ("dtype_tag", C.c_uint32), ("order", C.c_uint32),
-                ("evictable", C.c_uint32), ("n_pages", C.c_uint32)]
+                ("evictable", C.c_uint32), ("n_pages", C.c_uint32), ("consumers_left", C.c_uint32),
+                ("reserved", C.c_uint32)]
 
 
 _P = C.c_void_p
@@ -63,6 +64,7 @@ PROTOTYPES = {
     "t2i_store_destroy": (_S, [_P]),
     "t2i_put_batch": (_S, [_P, C.POINTER(PutDesc), _U32, _PU64, _P]),
     "t2i_get_batch": (_S, [_P, C.POINTER(GetDesc), _U32, C.POINTER(_S), _P]),
+    "t2i_get_batch_after": (_S, [_P, C.POINTER(GetDesc), _U32, C.POINTER(_S), _P, _P]),
     "t2i_free": (_S, [_P, _PU64, _U32]),
     "t2i_compact": (_S, [_P, _U64, _P, _PU64]),
     "t2i_store_stats": (_S, [_P, C.POINTER(Stats)]),

@@ -133,6 +133,12 @@ t2i_status Control::put(const t2i_put_desc* descs, uint32_t n, t2i_id* ids, std:
     std::vector<uint64_t> pinned;
     pinned.reserve(n);
     for (uint32_t i = 0; i < n; ++i) {
+        if (descs[i].reserved != 0) {
+            err_ = "put: reserved field must be 0";
+            return T2I_ERR_INVALID;
+        }
+    }
+    for (uint32_t i = 0; i < n; ++i) {
         const uint64_t np = pages_for(descs[i].nbytes);
         if (np > limit_pages_ || demand + np > limit_pages_) {
             err_ = "put: the batch needs more pages than the store has";
@@ -181,6 +187,7 @@ t2i_status Control::put(const t2i_put_desc* descs, uint32_t n, t2i_id* ids, std:
         o->dtype_tag = d.dtype_tag;
         o->order = d.order;
         o->evictable = d.evictable != 0;
+        o->consumers_left = d.consumers;
         o->group = group_for(d.group);
         const uint64_t np = pages_for(d.nbytes);
         o->pages.resize(np);
@@ -220,7 +227,7 @@ void Control::rollback_put(const t2i_id* ids, uint32_t n) {
 }
 
 t2i_status Control::get(const t2i_get_desc* descs, uint32_t n, t2i_status* per_item,
-                        std::vector<const Object*>* objs) {
+                        std::vector<const Object*>* objs, bool defer_release) {
     if (objs) objs->assign(n, nullptr);
     if (n == 0) return T2I_OK;
     if (!descs) {
@@ -264,9 +271,19 @@ t2i_status Control::get(const t2i_get_desc* descs, uint32_t n, t2i_status* per_i
         touch(o);
         counters_.gets++;
         counters_.bytes_got += o->nbytes;
+        if (o->consumers_left > 0 && --o->consumers_left == 0) pending_release_.push_back(o);
     }
     flush_touches();
+    if (!defer_release) release_pending();
     return T2I_OK;
+}
+
+void Control::release_pending() {
+    for (Object* o : pending_release_) {
+        counters_.reclaimed++;
+        release(o, false);
+    }
+    pending_release_.clear();
 }
 
 t2i_status Control::free(const t2i_id* ids, uint32_t n) {

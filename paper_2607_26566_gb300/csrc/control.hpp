@@ -16,6 +16,10 @@
 //     descriptor order; victims: least recent group first, then the highest
 //     `order`, then the highest id; groups named by the put are exempt, so are
 //     non-evictable objects; a put that cannot be satisfied evicts nothing;
+//   - an object put with k > 0 consumers is freed after its k-th successful
+//     get item (§5.3: reclaimed once no downstream consumer needs it); the
+//     objects a get brings to zero are freed at the end of that get, in the
+//     order of the items that brought them there;
 //   - compaction to `limit` pages moves the live pages numbered >= limit, in
 //     ascending order, to the lowest free pages below limit, then rebuilds the
 //     free stack from the free pages below limit so the lowest pops first.
@@ -41,6 +45,7 @@ struct Object {
     uint32_t dtype_tag = 0;
     uint32_t order = 0;
     bool evictable = false;
+    uint32_t consumers_left = 0;    // gets still expected before the store frees it (0 = none)
     Group* group = nullptr;
     size_t live_index = 0;          // position in Control::live_
     std::vector<uint32_t> pages;    // page list, in object byte order
@@ -95,10 +100,14 @@ class Control {
     t2i_status put(const t2i_put_desc* descs, uint32_t n, t2i_id* ids, std::vector<const Object*>* created);
     // Undo the put of freshly created objects (after a failed launch).
     void rollback_put(const t2i_id* ids, uint32_t n);
-    // get: validates every item (per_item nullable), then stamps recency.
-    // objs[i] receives the object of descs[i] on success. dst fields are not
-    // looked at here.
-    t2i_status get(const t2i_get_desc* descs, uint32_t n, t2i_status* per_item, std::vector<const Object*>* objs);
+    // get: validates every item (per_item nullable), then stamps recency and
+    // counts consumers. objs[i] receives the object of descs[i] on success.
+    // dst fields are not looked at here. Objects whose last consumer this was
+    // are freed at the end of the call, or, with defer_release, kept until
+    // release_pending() (the store frees them after packing its launches).
+    t2i_status get(const t2i_get_desc* descs, uint32_t n, t2i_status* per_item, std::vector<const Object*>* objs,
+                   bool defer_release = false);
+    void release_pending();
     t2i_status free(const t2i_id* ids, uint32_t n);
     // compact: plans, remaps and returns the moves (always filled).
     t2i_status compact(uint64_t limit_bytes, std::vector<t2i_move>* moves);
@@ -136,6 +145,7 @@ class Control {
     std::set<std::pair<uint64_t, Group*>> recency_;   // groups holding evictable objects
     std::vector<Group*> touched_;
     std::vector<t2i_id> last_evictions_;
+    std::vector<Object*> pending_release_;   // consumed to zero by the last get
     t2i_stats counters_{};
     std::string err_;
 };

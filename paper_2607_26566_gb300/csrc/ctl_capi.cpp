@@ -109,6 +109,8 @@ t2i_status t2i_ctl_object(const t2i_ctl* ctl, t2i_id id, t2i_object_info* info, 
         info->order = o->order;
         info->evictable = o->evictable ? 1u : 0u;
         info->n_pages = static_cast<uint32_t>(o->pages.size());
+        info->consumers_left = o->consumers_left;
+        info->reserved = 0;
     }
     if (pages) {
         const uint64_t k = o->pages.size() < cap ? o->pages.size() : cap;

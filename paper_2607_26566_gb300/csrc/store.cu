@@ -150,7 +150,8 @@ class Store {
     const std::string& error() const { return err_; }
 
     t2i_status put(const t2i_put_desc* descs, uint32_t n, t2i_id* ids, cudaStream_t stream);
-    t2i_status get(const t2i_get_desc* descs, uint32_t n, t2i_status* per_item, cudaStream_t stream);
+    t2i_status get(const t2i_get_desc* descs, uint32_t n, t2i_status* per_item, cudaStream_t stream,
+                   cudaEvent_t wait_event = nullptr);
     t2i_status free(const t2i_id* ids, uint32_t n) {
         t2i_status st = ctl_.free(ids, n);
         if (st != T2I_OK) err_ = ctl_.error();
@@ -458,7 +459,8 @@ t2i_status Store::put(const t2i_put_desc* descs, uint32_t n, t2i_id* ids, cudaSt
     return T2I_OK;
 }
 
-t2i_status Store::get(const t2i_get_desc* descs, uint32_t n, t2i_status* per_item, cudaStream_t stream) {
+t2i_status Store::get(const t2i_get_desc* descs, uint32_t n, t2i_status* per_item, cudaStream_t stream,
+                      cudaEvent_t wait_event) {
     if (n == 0) return T2I_OK;
     if (!descs) {
         err_ = "get: null descriptor array";
@@ -504,8 +506,9 @@ t2i_status Store::get(const t2i_get_desc* descs, uint32_t n, t2i_status* per_ite
                (first == T2I_ERR_INVALID && !why.empty() ? " (" + why + ")" : "");
         return first;
     }
-    // 2. LRU stamps
-    t2i_status st = ctl_.get(descs, n, per_item, &objs_);
+    // 2. LRU stamps and consumer counts (objects consumed to zero are freed
+    //    after their pages have been packed into this call's launches)
+    t2i_status st = ctl_.get(descs, n, per_item, &objs_, /*defer_release=*/true);
     if (st != T2I_OK) {
         err_ = ctl_.error();
         return st;
@@ -513,6 +516,14 @@ t2i_status Store::get(const t2i_get_desc* descs, uint32_t n, t2i_status* per_ite
     // 3. one gather launch for the batch (copies and casts together)
     DeviceGuard g(device_);
     order_after_last(stream);
+    if (wait_event) {
+        cudaError_t e = cudaStreamWaitEvent(stream, wait_event, 0);
+        if (e != cudaSuccess) {
+            err_ = std::string("get: cannot wait for the event: ") + cudaGetErrorString(e);
+            ctl_.release_pending();
+            return T2I_ERR_CUDA;
+        }
+    }
     segs_.clear();
     for (uint32_t i = 0; i < n; ++i) {
         const Object* o = objs_[i];
@@ -520,8 +531,9 @@ t2i_status Store::get(const t2i_get_desc* descs, uint32_t n, t2i_status* per_ite
         segs_.push_back({dev_dst[i], o->nbytes | (descs[i].cast ? kCastFlag : 0), o->pages.data(),
                          uint32_t(o->pages.size())});
     }
-    if (segs_.empty()) return T2I_OK;
-    return launch_segments<Mode::Get>(segs_, stream);
+    if (!segs_.empty()) st = launch_segments<Mode::Get>(segs_, stream);
+    ctl_.release_pending();
+    return st;
 }
 
 t2i_status Store::compact(uint64_t limit_bytes, cudaStream_t stream, uint64_t* moved) {
@@ -633,6 +645,12 @@ t2i_status t2i_put_batch(t2i_store* store, const t2i_put_desc* descs, uint32_t n
 t2i_status t2i_get_batch(t2i_store* store, const t2i_get_desc* descs, uint32_t n, t2i_status* per_item,
                          void* cuda_stream) {
     T2I_STORE_CALL(store, store->s->get(descs, n, per_item, static_cast<cudaStream_t>(cuda_stream)));
+}
+
+t2i_status t2i_get_batch_after(t2i_store* store, const t2i_get_desc* descs, uint32_t n, t2i_status* per_item,
+                               void* cuda_stream, void* wait_event) {
+    T2I_STORE_CALL(store, store->s->get(descs, n, per_item, static_cast<cudaStream_t>(cuda_stream),
+                                        static_cast<cudaEvent_t>(wait_event)));
 }
 
 t2i_status t2i_free(t2i_store* store, const t2i_id* ids, uint32_t n) {

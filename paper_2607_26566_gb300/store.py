@@ -15,7 +15,8 @@ import numpy as np
 from . import _lib as L
 
 PUT_DTYPE = np.dtype([("src", "<u8"), ("nbytes", "<u8"), ("src_is_host", "<u4"), ("dtype_tag", "<u4"),
-                      ("group", "<u8"), ("order", "<u4"), ("evictable", "<u4")])
+                      ("group", "<u8"), ("order", "<u4"), ("evictable", "<u4"), ("consumers", "<u4"),
+                      ("reserved", "<u4")])
 GET_DTYPE = np.dtype([("id", "<u8"), ("dst", "<u8"), ("dst_bytes", "<u8"), ("cast", "<u4"), ("reserved", "<u4")])
 MOVE_DTYPE = np.dtype([("src_page", "<u4"), ("dst_page", "<u4"), ("valid_bytes", "<u8")])
 assert PUT_DTYPE.itemsize == C.sizeof(L.PutDesc) and GET_DTYPE.itemsize == C.sizeof(L.GetDesc)
@@ -62,7 +63,8 @@ def _addrs(xs):
     return [_ptr(x) for x in xs]
 
 
-def put_descs(srcs, nbytes=None, src_is_host=0, dtype_tag=0, group=0, order=0, evictable=0) -> np.ndarray:
+def put_descs(srcs, nbytes=None, src_is_host=0, dtype_tag=0, group=0, order=0, evictable=0,
+              consumers=0) -> np.ndarray:
     """A put descriptor array. ``srcs``: tensors / arrays / addresses (an
     integer numpy array of addresses is taken as is; 0 or None reserves
     pages); scalars broadcast."""
@@ -75,6 +77,7 @@ def put_descs(srcs, nbytes=None, src_is_host=0, dtype_tag=0, group=0, order=0, e
     d["group"] = group
     d["order"] = order
     d["evictable"] = evictable
+    d["consumers"] = consumers
     return d
 
 
@@ -226,12 +229,18 @@ class Store:
                                      ids.ctypes.data_as(C.POINTER(C.c_uint64)), _stream(stream))
         return st, ids
 
-    def get_batch(self, descs: np.ndarray, stream=None, per_item: bool = True):
-        """(status, per-item statuses) -- t2i_get_batch."""
+    def get_batch(self, descs: np.ndarray, stream=None, per_item: bool = True, wait_event=None):
+        """(status, per-item statuses) -- t2i_get_batch, or t2i_get_batch_after
+        when ``wait_event`` (a torch.cuda.Event or a cudaEvent_t address) is given."""
         per = np.zeros(len(descs), np.int32) if per_item else None
-        st = self._lib.t2i_get_batch(self._h, _as(descs, L.GetDesc, GET_DTYPE), len(descs),
-                                     per.ctypes.data_as(C.POINTER(C.c_int32)) if per_item else None,
-                                     _stream(stream))
+        per_p = per.ctypes.data_as(C.POINTER(C.c_int32)) if per_item else None
+        if wait_event is None:
+            st = self._lib.t2i_get_batch(self._h, _as(descs, L.GetDesc, GET_DTYPE), len(descs), per_p,
+                                         _stream(stream))
+        else:
+            ev = wait_event if isinstance(wait_event, int) else int(wait_event.cuda_event)
+            st = self._lib.t2i_get_batch_after(self._h, _as(descs, L.GetDesc, GET_DTYPE), len(descs), per_p,
+                                               _stream(stream), ev)
         return st, per
 
     def free(self, ids) -> int:

@@ -14,12 +14,13 @@ def compare(ctl: Ctl, ora: OracleStore):
     s = ctl.stats()
     o = ora.summary()
     for k in ("used_pages", "free_pages", "limit_pages", "total_pages", "live_objects", "evictions",
-              "pages_moved", "bytes_moved", "bytes_put", "bytes_got", "misses"):
+              "pages_moved", "bytes_moved", "bytes_put", "bytes_got", "misses", "reclaimed"):
         assert s[k] == o[k], k
     for oid, obj in ora.objects.items():
         st, info, pages = ctl.object(oid)
         assert st == 0 and pages == obj.pages and info["nbytes"] == obj.nbytes
         assert info["group"] == obj.group and info["order"] == obj.order and info["evictable"] == int(obj.evictable)
+        assert info["consumers_left"] == obj.consumers_left
 
 
 def run_trace(seed, P, total_pages, n_ops, groups=4):
@@ -35,10 +36,11 @@ def run_trace(seed, P, total_pages, n_ops, groups=4):
             grp = g.integers(0, groups, k)
             order = g.integers(0, 6, k)
             ev = (g.random(k) < 0.6).astype(np.uint32)
-            d = put_descs([0] * k, nbytes=n, group=grp, order=order, evictable=ev)
+            cons = np.where(g.random(k) < 0.3, g.integers(1, 4, k), 0).astype(np.uint32)
+            d = put_descs([0] * k, nbytes=n, group=grp, order=order, evictable=ev, consumers=cons)
             st, ids = ctl.put(d)
-            ost, oids = ora.put_batch([PutItem(int(n[i]), None, 0, int(grp[i]), int(order[i]), bool(ev[i]))
-                                       for i in range(k)])
+            ost, oids = ora.put_batch([PutItem(int(n[i]), None, 0, int(grp[i]), int(order[i]), bool(ev[i]),
+                                               int(cons[i])) for i in range(k)])
             assert st == ost
             if st == 0:
                 assert list(ids) == oids

@@ -360,3 +360,38 @@ def test_compaction_moves_bytes_vs_oracle():
     s, moved = st.compact(pages * P)
     assert s == 0 and moved == 0 and ora.compact(pages * P)[0] == 0
     compare_meta(st, ora)
+
+
+def test_consumer_reclaim_and_deferred_get():
+    """An object put with 2 consumers is freed after its second get; a get
+    issued with a producer's event waits for it on the GPU (the producer runs
+    on a stream the store never saw, so only the event orders them)."""
+    P = 64 * 1024
+    st = make_store(64 * P, P)
+    s1, s2, s3 = torch.cuda.Stream(), torch.cuda.Stream(), torch.cuda.Stream()
+    x = torch.randint(0, 256, (5 * P + 3,), dtype=torch.uint8, device=DEV)
+    torch.cuda.synchronize()
+    s, (i,) = st.put_batch(put_descs([x], consumers=2), stream=s1)
+    assert s == 0 and st.ctl.object(int(i))[1]["consumers_left"] == 2
+    with torch.cuda.stream(s3):
+        torch.cuda._sleep(int(2.0e9 * 0.03))     # a 30 ms producer
+    ev = torch.cuda.Event()
+    ev.record(s3)
+    t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    out = torch.empty_like(x)
+    t0.record(s2)
+    s, _ = st.get_batch(get_descs([int(i)], [out]), stream=s2, wait_event=ev)
+    t1.record(s2)
+    assert s == 0
+    torch.cuda.synchronize()
+    assert t0.elapsed_time(t1) > 10.0, "the get did not wait for the producer's event"
+    assert torch.equal(out, x)
+    assert st.ctl.object(int(i))[1]["consumers_left"] == 1
+    out2 = torch.empty_like(x)
+    s, _ = st.get_batch(get_descs([int(i)], [out2]), stream=s2)
+    assert s == 0
+    torch.cuda.synchronize()
+    assert torch.equal(out2, x)
+    stats = st.stats()
+    assert stats["reclaimed"] == 1 and stats["live_objects"] == 0 and stats["used_pages"] == 0
+    assert st.get_batch(get_descs([int(i)], [out]))[0] == 3

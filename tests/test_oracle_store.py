@@ -75,7 +75,8 @@ def random_ops(seed, P, total_pages, n_ops, max_pages=3, check=True):
                 n = int(g.integers(0, max_pages * P + 1))
                 data = None if g.random() < 0.1 else g.integers(0, 256, n, dtype=np.uint8)
                 items.append(PutItem(n, data, group=int(g.integers(0, 3)), order=int(g.integers(0, 4)),
-                                     evictable=bool(g.random() < 0.5)))
+                                     evictable=bool(g.random() < 0.5),
+                                     consumers=int(g.integers(0, 3)) if g.random() < 0.3 else 0))
             free_before = s.free_pages()
             evictable_pages = sum(ceil_pages_by_counting(o.nbytes, P) for o in s.objects.values()
                                   if o.evictable and o.group not in {it.group for it in items})
@@ -99,6 +100,9 @@ def random_ops(seed, P, total_pages, n_ops, max_pages=3, check=True):
             for oid, out in zip(ids, outs):
                 if inputs[int(oid)] is not None:
                     assert np.array_equal(out, inputs[int(oid)])
+            for oid in ids:                      # consumed to zero: reclaimed
+                if int(oid) not in s.objects:
+                    inputs.pop(int(oid), None)
         elif r < 0.9 and inputs:
             ids = list(g.choice(list(inputs), size=min(len(inputs), int(g.integers(1, 3))), replace=False))
             assert s.free(ids) == OK
@@ -337,3 +341,37 @@ def test_planted_compaction_drops_bytes(monkeypatch):
         return st, moves
     monkeypatch.setattr(OracleStore, "compact", compact)
     assert _expect_failure(lambda: [random_ops(sd, 64, 16, 150) for sd in range(6)])
+
+
+def test_reclaim_by_consumer_count_hand_trace():
+    """Reading 9 (§5.3: reclaimed when no downstream consumer needs it)."""
+    P = 256
+    s = OracleStore(8 * P, P, paged_pool=True)
+    a, b, c = (np.full(300, v, np.uint8) for v in (1, 2, 3))
+    st, (ia, ib, ic) = s.put_batch([PutItem(300, a, consumers=2), PutItem(300, b, consumers=1),
+                                    PutItem(300, c)])
+    assert st == OK and s.pages_of(ia) == [0, 1] and s.pages_of(ib) == [2, 3]
+    st, _, outs = s.get_batch([ia, ib])
+    assert st == OK and np.array_equal(outs[1], b)
+    assert ib not in s.objects and s.free_stack[-2:] == [2, 3] and s.stats["reclaimed"] == 1
+    st, _, outs = s.get_batch([ia, ia])          # the last consumer may read twice in its batch
+    assert st == OK and np.array_equal(outs[0], a) and np.array_equal(outs[1], a)
+    assert ia not in s.objects and s.stats["reclaimed"] == 2
+    assert s.get_batch([ia])[0] == NOT_FOUND
+    st, _, (oc,) = s.get_batch([ic])
+    assert st == OK and ic in s.objects          # consumers = 0: only an explicit free
+    assert s.get_batch([ic, 999])[0] == NOT_FOUND and ic in s.objects  # a failed get consumes nothing
+    check_invariants(s, {ic: c})
+
+
+def test_planted_reclaim_before_last_consumer(monkeypatch):
+    orig = OracleStore.get_batch
+
+    def get_batch(self, ids, casts=None):
+        st, per, outs = orig(self, ids, casts)
+        for oid in list(self.objects):         # frees one consumer too early
+            if self.objects[oid].consumers_left == 1:
+                self._release(oid)
+        return st, per, outs
+    monkeypatch.setattr(OracleStore, "get_batch", get_batch)
+    assert _expect_failure(test_reclaim_by_consumer_count_hand_trace)
