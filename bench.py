@@ -51,6 +51,7 @@ def parse():
     p.add_argument("--requests", type=int, default=64)
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--no-cpu", action="store_true")
+    p.add_argument("--no-extras", action="store_true", help="skip the one-call and reclaim variants")
     p.add_argument("--sweep", action="store_true", help="also time B = 1 and B = 4")
     p.add_argument("--pool-gib", type=float, default=None, help="smaller pool (profiling small cases)")
     p.add_argument("--cpu-seconds", type=float, default=10.0, help="minimum CPU-baseline sample time")
@@ -152,7 +153,7 @@ class Handoff:
     once; a step issues raw C-ABI calls only."""
 
     def __init__(self, B: int, requests: int, device, host_buffers: bool = False, seed: int = 0,
-                 pool_bytes: int | None = None):
+                 pool_bytes: int | None = None, consumers: int = 0):
         import torch
 
         from paper_2607_26566_gb300 import Store, get_descs, put_descs
@@ -180,8 +181,12 @@ class Handoff:
             self.outputs.append(outs)
         torch.cuda.synchronize(device)
         self.ids = np.zeros(requests * self.n_obj, np.uint64)
+        # consumers = 1: every intermediate is reclaimed by the store after its
+        # one get (§5.3) and the step issues no free
+        self.consumers = consumers
         self.pd = [put_descs(ts, nbytes=[sp.nbytes for sp in self.specs], src_is_host=int(host_buffers),
-                             dtype_tag=[sp.dtype_tag for sp in self.specs]) for ts in self.inputs]
+                             dtype_tag=[sp.dtype_tag for sp in self.specs], consumers=consumers)
+                   for ts in self.inputs]
         casts = [1 if j == self.ci else 0 for j in range(self.n_obj)]
         self.gd = [get_descs(np.zeros(self.n_obj, np.uint64), outs, cast=casts) for outs in self.outputs]
         from paper_2607_26566_gb300 import _lib as L
@@ -221,9 +226,24 @@ class Handoff:
                 raise RuntimeError("get_batch: " + self.store.last_error())
         if ev is not None:
             ev[2].record()
-        st = lib.t2i_free(h, self.all_ids_p, len(self.ids))
-        if st:
-            raise RuntimeError("free: " + self.store.last_error())
+        if not self.consumers:
+            st = lib.t2i_free(h, self.all_ids_p, len(self.ids))
+            if st:
+                raise RuntimeError("free: " + self.store.last_error())
+
+    def step_one_call(self):
+        """The same step with one put_batch of all requests' objects and one
+        get_batch of all of them (descriptors built once)."""
+        if not hasattr(self, "pd_all"):
+            self.pd_all = np.concatenate(self.pd)
+            self.gd_all = np.concatenate(self.gd)
+        st, ids = self.store.put_batch(self.pd_all)
+        self.store.check(st)
+        self.gd_all["id"] = ids
+        st, _ = self.store.get_batch(self.gd_all, per_item=False)
+        self.store.check(st)
+        if not self.consumers:
+            self.store.check(self.store.free(ids))
 
     def verify(self):
         """get(put(x)) == x on every non-cast output after a step (cheap)."""
@@ -848,6 +868,31 @@ def main():
     del hw
     torch.cuda.empty_cache()
 
+    # the same bytes in one call per phase, and with reclaim by consumer count
+    extras = {}
+    if not args.no_extras:
+        hx = Handoff(B, args.requests, device, pool_bytes=pool_bytes)
+        stream = torch.cuda.current_stream(device)
+        for _ in range(3):
+            hx.step_one_call()
+        torch.cuda.synchronize(device)
+        a, z = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        for _ in range(10):
+            hx.step_one_call()
+        z.record(stream)
+        torch.cuda.synchronize(device)
+        extras["one_call_per_phase_gbs"] = round(hx.step_bytes * 10 / (a.elapsed_time(z) * 1e-3) / 1e9, 1)
+        hx.store.close()
+        del hx
+        hr = Handoff(B, args.requests, device, pool_bytes=pool_bytes, consumers=1)
+        ms_r, _, _, _ = time_handoff(hr, 10, 3, dist_ctx, per_kernel=False)
+        extras["reclaim_by_consumers_gbs"] = round(hr.step_bytes * 10 / (ms_r * 1e-3) / 1e9, 1)
+        extras["reclaimed_per_step"] = hr.store.stats()["reclaimed"] // 13
+        hr.store.close()
+        del hr
+        torch.cuda.empty_cache()
+
     sweep = {}
     if args.sweep:
         for Bs in (1, 4):
@@ -890,7 +935,7 @@ def main():
                        "parallelism": f"replicas x{dist_ctx.world}"},
             "hbm_frac": round(value / dist_ctx.world / peak, 4), "hbm_frac_nominal_8tbs": round(value / dist_ctx.world / 8000.0, 4),
             "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e, "gpu_launches": int(launches),
-            "clocks": clocks, "sweep": sweep or None, "rows": rows or None,
+            "clocks": clocks, "sweep": sweep or None, "extras": extras or None, "rows": rows or None,
         }
         print(json.dumps(line), flush=True)
     dist_ctx.close()
