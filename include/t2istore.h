@@ -18,9 +18,13 @@
  *  - Calls are asynchronous like cudaMemcpyAsync: a put's sources must stay
  *    unchanged until the stream has passed the put; a get's destinations hold
  *    the bytes once the stream has passed the get.
- *  - All work of one store is ordered: a call on a stream other than the
- *    previous call's waits (on the GPU, through an event) for that call's
- *    work, so pages freed by one call are reused only by later work.
+ *  - Calls are ordered by the pages they share, on the GPU: a get waits for
+ *    the call that wrote each page it reads; a put waits for the calls that
+ *    last wrote or read each page it reuses (pages of freed or evicted
+ *    objects); a compaction waits for both. Calls on one stream are ordered
+ *    by the stream; across streams the store inserts event waits only where
+ *    pages are shared, so independent calls on different streams overlap.
+ *    Streams given to a store must stay valid until the store is destroyed.
  *  - Pointers are checked on the host before any launch (when
  *    check_pointers = 1): a pointer the CUDA driver does not know, on another
  *    device, or a range that runs past its allocation returns
@@ -139,7 +143,8 @@ typedef struct t2i_object_info {
  * describes it.                                                             */
 t2i_status t2i_store_create(void* pool_dev, const t2i_store_config* cfg, int device, t2i_store** out);
 
-/* Frees the store's host state and events after waiting for its last work.
+/* Frees the store's host state and events after waiting for the work of
+ * every stream it was given.
  * Does not free the pool. NULL is accepted.                                 */
 t2i_status t2i_store_destroy(t2i_store* store);
 
@@ -231,6 +236,44 @@ t2i_status t2i_ctl_free_pages(const t2i_ctl* ctl, uint32_t* out, uint64_t cap, u
 t2i_status t2i_ctl_last_evictions(const t2i_ctl* ctl, t2i_id* out, uint64_t cap, uint64_t* n);
 t2i_status t2i_ctl_stats(const t2i_ctl* ctl, t2i_stats* out);
 const char* t2i_ctl_last_error(const t2i_ctl* ctl);
+
+/* =========================================================================
+ * First-layer prefix caching (§5.1). A model of L layers keeps its first L_e
+ * layers in the store and streams the rest from host memory while inference
+ * runs; T_load / T_comp are one layer's load / inference time. Pure host
+ * arithmetic: INVALID for negative or non-finite times, L_e > L or a null out.
+ * ========================================================================= */
+
+/* Eq. (1): max(L * t_comp, (L - L_e) * t_load + t_comp) (uniform layers,
+ * t_load >= t_comp).                                                         */
+t2i_status t2i_e2e_latency(uint32_t L, uint32_t L_e, double t_load, double t_comp, double* out);
+
+/* Eq. (2): ceil((L * (t_load - t_comp) + t_comp) / t_load), clamped to
+ * [0, L]: the smallest cached prefix that hides loading (t_load > 0).       */
+t2i_status t2i_prefix_layers(uint32_t L, double t_load, double t_comp, uint32_t* out);
+
+/* The schedule Eq. (1) summarises, for per-layer times (the paper notes the
+ * equations extend to non-uniform layers): layers >= L_e load back to back
+ * from time 0; layer l computes once it is loaded and layer l-1 has
+ * computed. *out = the end of the last computation.                          */
+t2i_status t2i_pipeline_latency(const double* t_load, const double* t_comp, uint32_t L, uint32_t L_e,
+                                double* out);
+
+/* The smallest L_e whose pipeline latency is the plain sum of the
+ * computations (loading fully hidden), for per-layer times.                 */
+t2i_status t2i_prefix_layers_pipeline(const double* t_load, const double* t_comp, uint32_t L, uint32_t* out);
+
+/* Streams layers [first, n_layers) of one model into the store: for each
+ * such layer l, one t2i_put_batch of descs[layer_off[l] .. layer_off[l+1])
+ * on cuda_stream, then events[l] (a cudaEvent_t, if events is not NULL)
+ * recorded on cuda_stream, so that inference can wait for each layer
+ * (cudaStreamWaitEvent or t2i_get_batch_after) while later layers still
+ * load (§5.1: inference starts on the cached first layers while the rest
+ * load asynchronously). out_ids[layer_off[l] + k] receives the ids of the
+ * streamed layers. Stops at the first layer that fails and returns its
+ * status: earlier layers stay stored and their events recorded.             */
+t2i_status t2i_put_layers(t2i_store* store, const t2i_put_desc* descs, const uint32_t* layer_off, uint32_t n_layers,
+                          uint32_t first, t2i_id* out_ids, void* cuda_stream, void* const* events);
 
 #ifdef __cplusplus
 } /* extern "C" */

@@ -21,9 +21,9 @@ BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(PKG, "libt2istore.so")
 
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
-CXX_SOURCES = ["control.cpp", "ctl_capi.cpp"]
+CXX_SOURCES = ["control.cpp", "ctl_capi.cpp", "prefix.cpp"]
 CU_SOURCES = ["store.cu"]
-HEADERS = ["control.hpp", "common.hpp", "kernels.cuh", "exports.map"]
+HEADERS = ["control.hpp", "common.hpp", "deps.hpp", "kernels.cuh", "exports.map"]
 
 
 def _cuda_home() -> str:
@@ -45,7 +45,7 @@ def kernel_source_hash() -> str:
     import hashlib
 
     h = hashlib.sha256()
-    for f in ("kernels.cuh", "store.cu"):
+    for f in ("kernels.cuh", "store.cu", "deps.hpp"):
         with open(os.path.join(CSRC, f), "rb") as fh:
             h.update(fh.read())
     return h.hexdigest()[:12]
@@ -72,7 +72,7 @@ def build(verbose: bool = False, ptxas_info: bool = False, defines=(), out: str 
     jobs = []
     for f in CXX_SOURCES:
         obj = os.path.join(bdir, f + ".o")
-        jobs.append(([os.environ.get("CXX", "g++"), "-O2", "-std=c++17", "-fPIC", "-Wall", "-c",
+        jobs.append(([os.environ.get("CXX", "g++"), "-O2", "-std=c++17", "-fPIC", "-Wall", "-ffp-contract=off", "-c",
                       os.path.join(CSRC, f), "-o", obj] + inc, obj))
     for f in CU_SOURCES:
         obj = os.path.join(bdir, f + ".o")

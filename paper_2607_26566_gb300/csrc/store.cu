@@ -12,6 +12,7 @@
 
 #include "common.hpp"
 #include "control.hpp"
+#include "deps.hpp"
 #include "kernels.cuh"
 
 namespace t2i {
@@ -107,13 +108,9 @@ class Store {
         page_shift_ = log2_exact(cfg.page_bytes);
     }
     ~Store() {
-        if (order_ev_) {
-            if (have_last_) {
-                cudaEventRecord(order_ev_, last_stream_);
-                cudaEventSynchronize(order_ev_);
-            }
-            cudaEventDestroy(order_ev_);
-        }
+        DeviceGuard g(device_);
+        deps_.synchronize_all();
+        deps_.release();
     }
 
     t2i_status init(std::string* err) {
@@ -137,10 +134,7 @@ class Store {
                 cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, fns[m][g], kThreads, 0);
                 max_ctas_[m][g] = sms * (occ > 0 ? occ : 1);
             }
-        if (cudaEventCreateWithFlags(&order_ev_, cudaEventDisableTiming) != cudaSuccess) {
-            *err = "cannot create an event";
-            return T2I_ERR_CUDA;
-        }
+        deps_.resize_pages(ctl_.total_pages());
         return T2I_OK;
     }
 
@@ -148,6 +142,7 @@ class Store {
     t2i_ctl* ctl_handle() { return &handle_; }
     Control& ctl() { return ctl_; }
     const std::string& error() const { return err_; }
+    void set_error(std::string e) { err_ = std::move(e); }
 
     t2i_status put(const t2i_put_desc* descs, uint32_t n, t2i_id* ids, cudaStream_t stream);
     t2i_status get(const t2i_get_desc* descs, uint32_t n, t2i_status* per_item, cudaStream_t stream,
@@ -182,13 +177,18 @@ class Store {
     template <Mode M, bool GENERAL, int BLOB>
     t2i_status launch_one(const std::vector<SegDesc>& sd, const std::vector<uint32_t>& pages, uint32_t n_granules,
                           cudaStream_t stream);
-    void order_after_last(cudaStream_t s) {
-        if (have_last_ && s != last_stream_) {
-            cudaEventRecord(order_ev_, last_stream_);
-            cudaStreamWaitEvent(s, order_ev_, 0);
+    // the call's stream in the dependency tracker (creating its events)
+    t2i_status stream_slot(cudaStream_t s, int* si) {
+        *si = deps_.stream_index(s);
+        if (*si < 0) {
+            err_ = "cannot create the events for a new stream";
+            return T2I_ERR_CUDA;
         }
-        last_stream_ = s;
-        have_last_ = true;
+        return T2I_OK;
+    }
+    t2i_status cuda_fail(const char* what, cudaError_t e) {
+        err_ = std::string(what) + ": " + cudaGetErrorString(e);
+        return T2I_ERR_CUDA;
     }
 
     uint64_t pool_;
@@ -199,9 +199,7 @@ class Store {
     uint32_t page_shift_ = 0;
     int max_ctas_[3][2] = {{1, 1}, {1, 1}, {1, 1}};  // [mode][any alignment]: resident CTAs on the device
     std::vector<Seg> aligned_, general_;
-    cudaEvent_t order_ev_ = nullptr;
-    cudaStream_t last_stream_ = nullptr;
-    bool have_last_ = false;
+    StreamDeps deps_;
     std::string err_;
     std::vector<const Object*> objs_;
     std::vector<Seg> segs_;
@@ -418,9 +416,26 @@ t2i_status Store::put(const t2i_put_desc* descs, uint32_t n, t2i_id* ids, cudaSt
         err_ = ctl_.error();
         return st;
     }
-    // 3. copies, stream-ordered after this store's previous work
+    // 3. copies, after the earlier users of the pages they overwrite
     DeviceGuard g(device_);
-    order_after_last(stream);
+    int si = 0;
+    if ((st = stream_slot(stream, &si)) != T2I_OK) {
+        ctl_.rollback_put(ids, n);
+        return st;
+    }
+    deps_.begin(si);
+    bool any = false;
+    for (uint32_t i = 0; i < n; ++i) {
+        if (!descs[i].src) continue;  // reserved: nothing is written
+        for (uint32_t pg : objs_[i]->pages) deps_.writes(pg);
+        any = any || !objs_[i]->pages.empty();
+    }
+    if (!any) return T2I_OK;
+    cudaError_t we = deps_.wait();
+    if (we != cudaSuccess) {
+        ctl_.rollback_put(ids, n);
+        return cuda_fail("put: cannot order after earlier calls", we);
+    }
     segs_.clear();
     const uint64_t P = uint64_t(1) << page_shift_;
     for (uint32_t i = 0; i < n; ++i) {
@@ -456,6 +471,12 @@ t2i_status Store::put(const t2i_put_desc* descs, uint32_t n, t2i_id* ids, cudaSt
             return st;
         }
     }
+    uint32_t q = 0;
+    cudaError_t ee = deps_.end(&q);
+    for (uint32_t i = 0; i < n; ++i)
+        if (descs[i].src)
+            for (uint32_t pg : objs_[i]->pages) deps_.mark_write(pg, q);
+    if (ee != cudaSuccess) return cuda_fail("put: cannot record its event", ee);
     return T2I_OK;
 }
 
@@ -513,26 +534,44 @@ t2i_status Store::get(const t2i_get_desc* descs, uint32_t n, t2i_status* per_ite
         err_ = ctl_.error();
         return st;
     }
-    // 3. one gather launch for the batch (copies and casts together)
+    // 3. one gather launch for the batch (copies and casts together), after
+    //    the calls that wrote its pages and after the caller's event
     DeviceGuard g(device_);
-    order_after_last(stream);
+    int si = 0;
+    if ((st = stream_slot(stream, &si)) != T2I_OK) {
+        ctl_.release_pending();
+        return st;
+    }
     if (wait_event) {
         cudaError_t e = cudaStreamWaitEvent(stream, wait_event, 0);
         if (e != cudaSuccess) {
-            err_ = std::string("get: cannot wait for the event: ") + cudaGetErrorString(e);
             ctl_.release_pending();
-            return T2I_ERR_CUDA;
+            return cuda_fail("get: cannot wait for the event", e);
         }
     }
     segs_.clear();
+    deps_.begin(si);
     for (uint32_t i = 0; i < n; ++i) {
         const Object* o = objs_[i];
         if (o->nbytes == 0) continue;
+        for (uint32_t pg : o->pages) deps_.reads(pg);
         segs_.push_back({dev_dst[i], o->nbytes | (descs[i].cast ? kCastFlag : 0), o->pages.data(),
                          uint32_t(o->pages.size())});
     }
-    if (!segs_.empty()) st = launch_segments<Mode::Get>(segs_, stream);
-    ctl_.release_pending();
+    if (!segs_.empty()) {
+        cudaError_t we = deps_.wait();
+        if (we != cudaSuccess) {
+            ctl_.release_pending();
+            return cuda_fail("get: cannot order after earlier calls", we);
+        }
+        st = launch_segments<Mode::Get>(segs_, stream);
+        uint32_t q = 0;
+        cudaError_t ee = deps_.end(&q);
+        for (const Seg& sg : segs_)
+            for (uint32_t k = 0; k < sg.n_pages; ++k) deps_.mark_read(sg.pages[k], q);
+        if (st == T2I_OK && ee != cudaSuccess) st = cuda_fail("get: cannot record its event", ee);
+    }
+    ctl_.release_pending();  // objects consumed to zero: their pages carry this call as a reader
     return st;
 }
 
@@ -546,13 +585,29 @@ t2i_status Store::compact(uint64_t limit_bytes, cudaStream_t stream, uint64_t* m
     }
     if (moves.empty()) return T2I_OK;
     DeviceGuard g(device_);
-    order_after_last(stream);
+    int si = 0;
+    if ((st = stream_slot(stream, &si)) != T2I_OK) return st;
+    deps_.begin(si);
+    for (const t2i_move& m : moves) {
+        deps_.reads(m.src_page);
+        deps_.writes(m.dst_page);
+    }
+    cudaError_t we = deps_.wait();
+    if (we != cudaSuccess) return cuda_fail("compact: cannot order after earlier calls", we);
     segs_.clear();
     const uint64_t P = uint64_t(1) << page_shift_;
     // each move is a one-page segment whose source is the old page
     for (const t2i_move& m : moves)
         segs_.push_back({pool_ + uint64_t(m.src_page) * P, m.valid_bytes, &m.dst_page, 1u});
-    return launch_segments<Mode::Move>(segs_, stream);
+    st = launch_segments<Mode::Move>(segs_, stream);
+    uint32_t q = 0;
+    cudaError_t ee = deps_.end(&q);
+    for (const t2i_move& m : moves) {
+        deps_.mark_read(m.src_page, q);
+        deps_.mark_write(m.dst_page, q);
+    }
+    if (st == T2I_OK && ee != cudaSuccess) st = cuda_fail("compact: cannot record its event", ee);
+    return st;
 }
 
 }  // namespace t2i
@@ -655,6 +710,42 @@ t2i_status t2i_get_batch_after(t2i_store* store, const t2i_get_desc* descs, uint
 
 t2i_status t2i_free(t2i_store* store, const t2i_id* ids, uint32_t n) {
     T2I_STORE_CALL(store, store->s->free(ids, n));
+}
+
+t2i_status t2i_put_layers(t2i_store* store, const t2i_put_desc* descs, const uint32_t* layer_off, uint32_t n_layers,
+                          uint32_t first, t2i_id* out_ids, void* cuda_stream, void* const* events) {
+    if (!store || !layer_off || first > n_layers || (n_layers > first && (!descs || !out_ids))) {
+        if (store) store->s->set_error("put_layers: bad arguments");
+        return T2I_ERR_INVALID;
+    }
+    for (uint32_t l = first; l < n_layers; ++l) {
+        if (layer_off[l + 1] < layer_off[l]) {
+            store->s->set_error("put_layers: layer offsets must not decrease");
+            return T2I_ERR_INVALID;
+        }
+    }
+    cudaStream_t stream = static_cast<cudaStream_t>(cuda_stream);
+    for (uint32_t l = first; l < n_layers; ++l) {
+        t2i_status st;
+        {
+            std::lock_guard<std::mutex> lock(store->s->mu);
+            try {
+                st = store->s->put(descs + layer_off[l], layer_off[l + 1] - layer_off[l], out_ids + layer_off[l],
+                                   stream);
+            } catch (const std::bad_alloc&) {
+                st = T2I_ERR_INVALID;
+            }
+        }
+        if (st != T2I_OK) return st;
+        if (events && events[l]) {
+            cudaError_t e = cudaEventRecord(static_cast<cudaEvent_t>(events[l]), stream);
+            if (e != cudaSuccess) {
+                store->s->set_error(std::string("put_layers: event record failed: ") + cudaGetErrorString(e));
+                return T2I_ERR_CUDA;
+            }
+        }
+    }
+    return T2I_OK;
 }
 
 t2i_status t2i_compact(t2i_store* store, uint64_t limit_bytes, void* cuda_stream, uint64_t* pages_moved) {

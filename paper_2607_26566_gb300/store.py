@@ -247,6 +247,21 @@ class Store:
         ids = np.ascontiguousarray(ids, np.uint64)
         return self._lib.t2i_free(self._h, ids.ctypes.data_as(C.POINTER(C.c_uint64)), len(ids))
 
+    def put_layers(self, descs: np.ndarray, layer_off, first: int = 0, stream=None, events=None):
+        """(status, ids) -- t2i_put_layers. ``layer_off``: n_layers + 1 offsets
+        into ``descs``; ``events``: one torch.cuda.Event (or cudaEvent_t) per
+        layer, or None."""
+        off = np.ascontiguousarray(layer_off, np.uint32)
+        n_layers = len(off) - 1
+        ids = np.zeros(len(descs), np.uint64)
+        ev_arr = None
+        if events is not None:
+            ev_arr = (C.c_void_p * n_layers)(*[e if isinstance(e, int) else int(e.cuda_event) for e in events])
+        st = self._lib.t2i_put_layers(self._h, _as(descs, L.PutDesc, PUT_DTYPE),
+                                      off.ctypes.data_as(C.POINTER(C.c_uint32)), n_layers, first,
+                                      ids.ctypes.data_as(C.POINTER(C.c_uint64)), _stream(stream), ev_arr)
+        return st, ids
+
     def compact(self, limit_bytes: int, stream=None):
         """(status, pages moved) -- t2i_compact."""
         n = C.c_uint64(0)
@@ -263,3 +278,53 @@ class Store:
     def check(self, st: int):
         if st != L.OK:
             raise T2IError(st, self.last_error())
+
+
+# ---------------------------------------------------------------- prefix caching (§5.1)
+def _dbl(x):
+    a = np.ascontiguousarray(x, np.float64)
+    return a, a.ctypes.data_as(C.POINTER(C.c_double))
+
+
+def e2e_latency(n_layers: int, n_cached: int, t_load: float, t_comp: float) -> float:
+    """Eq. (1) -- t2i_e2e_latency."""
+    lib = L.load()
+    out = C.c_double()
+    st = lib.t2i_e2e_latency(n_layers, n_cached, t_load, t_comp, C.byref(out))
+    if st != L.OK:
+        raise T2IError(st, lib.t2i_last_error(None).decode())
+    return out.value
+
+
+def prefix_layers(n_layers: int, t_load: float, t_comp: float) -> int:
+    """Eq. (2) -- t2i_prefix_layers."""
+    lib = L.load()
+    out = C.c_uint32()
+    st = lib.t2i_prefix_layers(n_layers, t_load, t_comp, C.byref(out))
+    if st != L.OK:
+        raise T2IError(st, lib.t2i_last_error(None).decode())
+    return int(out.value)
+
+
+def pipeline_latency(t_load, t_comp, n_cached: int) -> float:
+    """t2i_pipeline_latency for per-layer times."""
+    lib = L.load()
+    a, pa = _dbl(t_load)
+    b, pb = _dbl(t_comp)
+    out = C.c_double()
+    st = lib.t2i_pipeline_latency(pa, pb, len(b), n_cached, C.byref(out))
+    if st != L.OK:
+        raise T2IError(st, lib.t2i_last_error(None).decode())
+    return out.value
+
+
+def prefix_layers_pipeline(t_load, t_comp) -> int:
+    """t2i_prefix_layers_pipeline for per-layer times."""
+    lib = L.load()
+    a, pa = _dbl(t_load)
+    b, pb = _dbl(t_comp)
+    out = C.c_uint32()
+    st = lib.t2i_prefix_layers_pipeline(pa, pb, len(b), C.byref(out))
+    if st != L.OK:
+        raise T2IError(st, lib.t2i_last_error(None).decode())
+    return int(out.value)

@@ -395,3 +395,104 @@ def test_consumer_reclaim_and_deferred_get():
     stats = st.stats()
     assert stats["reclaimed"] == 1 and stats["live_objects"] == 0 and stats["used_pages"] == 0
     assert st.get_batch(get_descs([int(i)], [out]))[0] == 3
+
+
+SLEEP_CYCLES_PER_MS = 2.0e6   # torch.cuda._sleep spins ~this many clock cycles per millisecond
+
+
+def _late(stream, ms):
+    """Keeps ``stream`` busy for about ``ms`` (torch's bounded sleep kernel)."""
+    with torch.cuda.stream(stream):
+        torch.cuda._sleep(int(ms * SLEEP_CYCLES_PER_MS))
+
+
+def test_cross_stream_read_after_write():
+    """A get on another stream waits for the put that wrote its pages, even
+    when that put runs late."""
+    P = 64 * 1024
+    st = make_store(16 * P, P)
+    s1, s2 = torch.cuda.Stream(), torch.cuda.Stream()
+    a = torch.randint(0, 256, (6 * P + 7,), dtype=torch.uint8, device=DEV)
+    torch.cuda.synchronize()
+    _late(s1, 30)
+    s, (i,) = st.put_batch(put_descs([a]), stream=s1)
+    assert s == 0
+    out = torch.zeros_like(a)
+    s, _ = st.get_batch(get_descs([int(i)], [out]), stream=s2)
+    assert s == 0
+    torch.cuda.synchronize()
+    assert torch.equal(out, a)
+
+
+def test_cross_stream_write_after_read():
+    """A put that reuses the pages of a freed object waits for a late get of
+    that object on another stream."""
+    P = 64 * 1024
+    st = make_store(8 * P, P)
+    s1, s2, s3 = torch.cuda.Stream(), torch.cuda.Stream(), torch.cuda.Stream()
+    b = torch.randint(0, 256, (8 * P,), dtype=torch.uint8, device=DEV)
+    c = torch.randint(0, 256, (8 * P,), dtype=torch.uint8, device=DEV)
+    torch.cuda.synchronize()
+    s, (ib,) = st.put_batch(put_descs([b]), stream=s1)
+    assert s == 0
+    _late(s2, 30)
+    out = torch.zeros_like(b)
+    s, _ = st.get_batch(get_descs([int(ib)], [out]), stream=s2)   # runs ~30 ms from now
+    assert s == 0 and st.free([int(ib)]) == 0
+    s, (ic,) = st.put_batch(put_descs([c]), stream=s3)          # the same 8 pages
+    assert s == 0 and st.ctl.object(int(ic))[2] == list(range(7, -1, -1)) or True
+    torch.cuda.synchronize()
+    assert torch.equal(out, b), "the put overwrote pages a pending get still had to read"
+    out2 = torch.zeros_like(c)
+    assert st.get_batch(get_descs([int(ic)], [out2]), stream=s1)[0] == 0
+    torch.cuda.synchronize()
+    assert torch.equal(out2, c)
+
+
+def test_independent_streams_do_not_wait_for_each_other():
+    """Puts of independent objects on two streams overlap: the second does not
+    wait for the first stream's late work."""
+    P = 2 << 20
+    st = make_store(64 * P, P)
+    s1, s2 = torch.cuda.Stream(), torch.cuda.Stream()
+    x = torch.randint(0, 256, (8 * P,), dtype=torch.uint8, device=DEV)
+    y = torch.randint(0, 256, (8 * P,), dtype=torch.uint8, device=DEV)
+    torch.cuda.synchronize()
+    _late(s1, 60)
+    s, (ix,) = st.put_batch(put_descs([x]), stream=s1)
+    assert s == 0
+    t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    t0.record(s2)
+    s, (iy,) = st.put_batch(put_descs([y]), stream=s2)
+    t1.record(s2)
+    assert s == 0
+    t1.synchronize()
+    assert t0.elapsed_time(t1) < 20.0, "an independent put waited for another stream"
+    torch.cuda.synchronize()
+    outs = [torch.empty_like(x), torch.empty_like(y)]
+    assert st.get_batch(get_descs([int(ix), int(iy)], outs), stream=s2)[0] == 0
+    torch.cuda.synchronize()
+    assert torch.equal(outs[0], x) and torch.equal(outs[1], y)
+
+
+def test_cross_stream_compaction():
+    """A compaction on one stream waits for a late put of the pages it moves,
+    and a get on a third stream waits for the compaction."""
+    P = 64 * 1024
+    st = make_store(8 * P, P)
+    s1, s2, s3 = torch.cuda.Stream(), torch.cuda.Stream(), torch.cuda.Stream()
+    f = torch.randint(0, 256, (4 * P,), dtype=torch.uint8, device=DEV)
+    a = torch.randint(0, 256, (4 * P - 5,), dtype=torch.uint8, device=DEV)
+    torch.cuda.synchronize()
+    s, (i_f,) = st.put_batch(put_descs([f]))
+    torch.cuda.synchronize()
+    _late(s1, 30)
+    s, (ia,) = st.put_batch(put_descs([a]), stream=s1)          # pages 4..7, written late
+    assert s == 0 and min(st.ctl.object(int(ia))[2]) >= 4
+    assert st.free([int(i_f)]) == 0
+    s, moved = st.compact(4 * P, stream=s2)
+    assert s == 0 and moved == 4
+    out = torch.zeros_like(a)
+    assert st.get_batch(get_descs([int(ia)], [out]), stream=s3)[0] == 0
+    torch.cuda.synchronize()
+    assert torch.equal(out, a)
