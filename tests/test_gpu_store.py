@@ -440,7 +440,7 @@ def test_cross_stream_write_after_read():
     s, _ = st.get_batch(get_descs([int(ib)], [out]), stream=s2)   # runs ~30 ms from now
     assert s == 0 and st.free([int(ib)]) == 0
     s, (ic,) = st.put_batch(put_descs([c]), stream=s3)          # the same 8 pages
-    assert s == 0 and st.ctl.object(int(ic))[2] == list(range(7, -1, -1)) or True
+    assert s == 0 and sorted(st.ctl.object(int(ic))[2]) == list(range(8))
     torch.cuda.synchronize()
     assert torch.equal(out, b), "the put overwrote pages a pending get still had to read"
     out2 = torch.zeros_like(c)
