@@ -55,7 +55,7 @@ def parse():
     p.add_argument("--sweep", action="store_true", help="also time B = 1 and B = 4")
     p.add_argument("--pool-gib", type=float, default=None, help="smaller pool (profiling small cases)")
     p.add_argument("--cpu-seconds", type=float, default=10.0, help="minimum CPU-baseline sample time")
-    p.add_argument("--rows", default="weights,adapters,compaction",
+    p.add_argument("--rows", default="weights,adapters,compaction,prefix",
                    help="other hot-path rows timed in the same run (comma list, or 'none')")
     p.add_argument("--adapter-calls", type=int, default=10_000)
     p.add_argument("--rows-only", action="store_true", help="skip the handoff headline (profiling a row)")
@@ -739,6 +739,144 @@ def time_compaction(device, reps: int = 2, pool_gib: int | None = None):
     return out
 
 
+# ----------------------------------------------------------------------------- prefix caching
+class PrefixPipeline:
+    """First-layer prefix caching (§5.1) on the 57-block DiT: the first L_e
+    blocks stay in the store; on a request the rest stream from pinned host
+    memory (copy engine, one t2i_put_layers on a load stream, an event per
+    block) while a compute stream takes each block out of the store
+    (t2i_get_batch_after on its event) and runs a synthetic inference of
+    T_comp per block (torch's bounded sleep kernel)."""
+
+    def __init__(self, device, n_blocks: int | None = None, load_to_comp: float = 3.2, seed: int = 0):
+        import torch
+
+        from paper_2607_26566_gb300 import get_descs
+
+        self.torch = torch
+        self.device = device
+        self.wr = WeightRestore(device, seed=seed, h2d_mode=1, n_blocks=n_blocks)
+        self.store = self.wr.store
+        self.L = len(self.wr.layout)
+        self.off = np.zeros(self.L + 1, np.uint32)
+        for b, d in enumerate(self.wr.pd):
+            self.off[b + 1] = self.off[b] + len(d)
+        self.descs = np.concatenate(self.wr.pd)
+        self.work = torch.empty(max(t for t, _ in self.wr.layout), dtype=torch.uint8, device=device)
+        self.s_load = torch.cuda.Stream(device)
+        self.s_comp = torch.cuda.Stream(device)
+        self.ids = np.zeros(len(self.descs), np.uint64)
+        self.get_descs = get_descs
+        self.load_to_comp = load_to_comp
+        self.cycles_per_ms = None
+
+    def _layer_gd(self, b):
+        lo, hi = int(self.off[b]), int(self.off[b + 1])
+        rel = [0]
+        for n in self.descs["nbytes"][lo:hi][:-1]:
+            rel.append(rel[-1] + int((int(n) + 255) // 256 * 256))
+        return self.get_descs(self.ids[lo:hi], self.work.data_ptr() + np.array(rel, np.uint64),
+                              dst_bytes=self.descs["nbytes"][lo:hi])
+
+    def free_all(self):
+        live = [int(i) for i in self.ids if int(i)]
+        if live:
+            self.store.check(self.store.free(live))
+        self.ids[:] = 0
+
+    def calibrate(self):
+        """Per-block load times (events between consecutive blocks of one
+        streamed load) and per-block get times; the sleep kernel's rate."""
+        torch = self.torch
+        self.free_all()
+        ev = [torch.cuda.Event(enable_timing=True) for _ in range(self.L + 1)]
+        ev[0].record(self.s_load)
+        st, ids = self.store.put_layers(self.descs, self.off, 0, stream=self.s_load, events=ev[1:])
+        self.store.check(st)
+        self.ids[:] = ids
+        torch.cuda.synchronize(self.device)
+        self.t_load = [ev[b].elapsed_time(ev[b + 1]) for b in range(self.L)]
+        g = [torch.cuda.Event(enable_timing=True) for _ in range(self.L + 1)]
+        g[0].record(self.s_comp)
+        for b in range(self.L):
+            self.store.check(self.store.get_batch(self._layer_gd(b), stream=self.s_comp, per_item=False)[0])
+            g[b + 1].record(self.s_comp)
+        torch.cuda.synchronize(self.device)
+        self.t_get = [g[b].elapsed_time(g[b + 1]) for b in range(self.L)]
+        a, z = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        with torch.cuda.stream(self.s_comp):
+            a.record()
+            torch.cuda._sleep(int(20e6))
+            z.record()
+        torch.cuda.synchronize(self.device)
+        self.cycles_per_ms = 20e6 / a.elapsed_time(z)
+        mean_load = sum(self.t_load) / self.L
+        self.t_sleep = mean_load / self.load_to_comp
+        self.free_all()
+
+    def request(self, L_e: int):
+        """One request with the first L_e blocks cached; returns ms."""
+        torch = self.torch
+        self.free_all()
+        st, ids = self.store.put_layers(self.descs, self.off[:L_e + 1], 0, stream=self.s_comp)
+        self.store.check(st)
+        self.ids[:int(self.off[L_e])] = ids
+        torch.cuda.synchronize(self.device)
+        ev = [torch.cuda.Event() for _ in range(self.L)]
+        t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        # the request arrives at t0: loading and inference start together (a
+        # 20 ms gate on the compute stream lets the host queue everything first)
+        with torch.cuda.stream(self.s_comp):
+            torch.cuda._sleep(int(20 * self.cycles_per_ms))
+        t0.record(self.s_comp)
+        self.s_load.wait_event(t0)
+        st, ids = self.store.put_layers(self.descs, self.off, L_e, stream=self.s_load, events=ev)
+        self.store.check(st)
+        lo = int(self.off[L_e])
+        self.ids[lo:] = ids[lo:]
+        cycles = int(self.t_sleep * self.cycles_per_ms)
+        for b in range(self.L):
+            self.store.check(self.store.get_batch(self._layer_gd(b), stream=self.s_comp, per_item=False,
+                                                  wait_event=ev[b] if b >= L_e else None)[0])
+            with torch.cuda.stream(self.s_comp):
+                torch.cuda._sleep(cycles)
+        t1.record(self.s_comp)
+        torch.cuda.synchronize(self.device)
+        return t0.elapsed_time(t1)
+
+    def close(self):
+        self.wr.close()
+
+
+def time_prefix(device, n_blocks: int | None = None, reps: int = 2):
+    from paper_2607_26566_gb300 import e2e_latency, pipeline_latency, prefix_layers, prefix_layers_pipeline
+
+    pp = PrefixPipeline(device, n_blocks=n_blocks)
+    pp.calibrate()
+    L = pp.L
+    comp = [pp.t_sleep + g for g in pp.t_get]          # per block on the compute stream
+    le_star = prefix_layers_pipeline(pp.t_load, comp)
+    mean_load, mean_comp = sum(pp.t_load) / L, sum(comp) / L
+    le_eq2 = prefix_layers(L, mean_load, mean_comp)
+    out = {"workload": f"prefix caching: {L}-block DiT weights from pinned host (copy engine), "
+                       f"T_load/T_comp = {pp.load_to_comp} per block on average",
+           "blocks": L, "t_load_ms_mean": round(mean_load, 4), "t_comp_ms_mean": round(mean_comp, 4),
+           "prefix_pipeline": le_star, "prefix_eq2": le_eq2, "compute_only_ms": round(sum(comp), 3), "runs": {}}
+    for L_e in sorted({0, le_star // 2, le_star, L}):
+        ms = min(pp.request(L_e) for _ in range(reps))
+        out["runs"][str(L_e)] = {"measured_ms": round(ms, 3),
+                                 "pipeline_model_ms": round(pipeline_latency(pp.t_load, comp, L_e), 3),
+                                 "eq1_ms": round(e2e_latency(L, L_e, mean_load, mean_comp), 3),
+                                 "exposed_loading_ms": round(ms - sum(comp), 3)}
+    r = out["runs"]
+    if "0" in r and str(le_star) in r:
+        base = r["0"]["exposed_loading_ms"]
+        for k in r:
+            r[k]["loading_reduction_vs_ppl0"] = round(1 - r[k]["exposed_loading_ms"] / base, 3) if base > 0 else None
+    pp.close()
+    return out
+
+
 # ----------------------------------------------------------------------------- CPU (oracle)
 def oracle_sample(B: int, n_requests: int, min_seconds: float = 0.0, max_steps: int = 1):
     """The oracle as it stands on the host: steps of the handoff workload (put
@@ -815,6 +953,8 @@ def run_rows(args, device, peak):
         rows["adapters"] = time_adapters(device, n_calls=args.adapter_calls)
     if "compaction" in wanted:
         rows["compaction"] = time_compaction(device, pool_gib=args.compaction_gib)
+    if "prefix" in wanted:
+        rows["prefix"] = time_prefix(device)
     for r in rows.values():
         for k in ("get_gbs", "gbs", "hit_gbs"):
             if k in r:

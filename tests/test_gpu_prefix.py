@@ -1,0 +1,71 @@
+"""Prefix caching with layer-streamed loading on the GPU (marked gpu): the
+blocks of a DiT stream into the store on a load stream with an event per
+block while a compute stream takes each block out after its event; every
+block's bytes arrive intact, and caching the first blocks shortens the
+request as the pipeline model says it should."""
+import numpy as np
+import pytest
+import torch
+
+import bench
+
+pytestmark = pytest.mark.gpu
+DEV = torch.device("cuda", 0)
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _built(lib):
+    assert torch.cuda.is_available(), "GPU tests need a CUDA device"
+    yield
+
+
+def test_layer_streaming_bytes_and_overlap():
+    from paper_2607_26566_gb300 import pipeline_latency, prefix_layers_pipeline
+
+    pp = bench.PrefixPipeline(DEV, n_blocks=8)
+    pp.calibrate()
+    comp = [pp.t_sleep + g for g in pp.t_get]
+    le = prefix_layers_pipeline(pp.t_load, comp)
+    assert 0 < le < pp.L
+    t_none = pp.request(0)
+    # every block got during the request equals its pinned host bytes
+    for b in range(pp.L):
+        st, _ = pp.store.get_batch(pp._layer_gd(b), stream=pp.s_comp, per_item=False)
+        assert st == 0
+        torch.cuda.synchronize()
+        total, members = pp.wr.layout[b]
+        h = pp.wr.host[b]
+        for i, off in members:
+            n = pp.wr.specs[i].nbytes
+            assert torch.equal(pp.work[off:off + n].cpu(), h[off:off + n]), (b, i)
+    t_cached = pp.request(le)
+    # loading is hidden: the cached request is faster and close to the model
+    assert t_cached < t_none
+    model_none = pipeline_latency(pp.t_load, comp, 0)
+    assert abs(t_none - model_none) / model_none < 0.25
+    pp.close()
+
+
+def test_reverse_layer_eviction_keeps_the_prefix():
+    """Under pressure the last blocks of the least recently used model go
+    first (§5.3), so the cached prefix survives."""
+    from paper_2607_26566_gb300 import Store, put_descs
+
+    P = 2 << 20
+    pool = torch.empty(64 * P, dtype=torch.uint8, device=DEV)
+    st = Store(pool, P)
+    src = torch.randint(0, 256, (P,), dtype=torch.uint8, device=DEV)
+    # model 1: 10 layers of 4 pages each (40 pages), evictable
+    s, ids1 = st.put_batch(put_descs([src] * 40, nbytes=P, group=1, order=np.repeat(np.arange(10), 4),
+                                     evictable=1))
+    assert s == 0
+    # model 2 needs 40 pages: 24 are free, 16 must be evicted from model 1
+    s, _ = st.put_batch(put_descs([src] * 40, nbytes=P, group=2, order=np.repeat(np.arange(10), 4), evictable=1))
+    assert s == 0
+    evicted = st.ctl.last_evictions()
+    assert len(evicted) == 16
+    layers = sorted({int(np.repeat(np.arange(10), 4)[int(i) - 1]) for i in evicted})
+    assert layers == [6, 7, 8, 9]            # the last four layers, highest first
+    assert evicted[:4] == [40, 39, 38, 37]   # layer 9, highest id first
+    live = [int(i) for i in ids1 if st.ctl.object(int(i))[0] == 0]
+    assert live == list(range(1, 25))        # layers 0..5 kept
