@@ -820,7 +820,8 @@ class PrefixPipeline:
         self.free_all()
         st, ids = self.store.put_layers(self.descs, self.off[:L_e + 1], 0, stream=self.s_comp)
         self.store.check(st)
-        self.ids[:int(self.off[L_e])] = ids
+        n = int(self.off[L_e])
+        self.ids[:n] = ids[:n]
         torch.cuda.synchronize(self.device)
         ev = [torch.cuda.Event() for _ in range(self.L)]
         t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)

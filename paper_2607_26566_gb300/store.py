@@ -239,6 +239,8 @@ class Store:
                                          _stream(stream))
         else:
             ev = wait_event if isinstance(wait_event, int) else int(wait_event.cuda_event)
+            if not ev:
+                raise ValueError("wait_event has never been recorded")
             st = self._lib.t2i_get_batch_after(self._h, _as(descs, L.GetDesc, GET_DTYPE), len(descs), per_p,
                                                _stream(stream), ev)
         return st, per
@@ -256,7 +258,12 @@ class Store:
         ids = np.zeros(len(descs), np.uint64)
         ev_arr = None
         if events is not None:
-            ev_arr = (C.c_void_p * n_layers)(*[e if isinstance(e, int) else int(e.cuda_event) for e in events])
+            handles = []
+            for e in events:
+                if not isinstance(e, int) and not e.cuda_event:
+                    e.record(stream if stream is not None and not isinstance(stream, int) else None)  # creates it
+                handles.append(e if isinstance(e, int) else int(e.cuda_event))
+            ev_arr = (C.c_void_p * n_layers)(*handles)
         st = self._lib.t2i_put_layers(self._h, _as(descs, L.PutDesc, PUT_DTYPE),
                                       off.ctypes.data_as(C.POINTER(C.c_uint32)), n_layers, first,
                                       ids.ctypes.data_as(C.POINTER(C.c_uint64)), _stream(stream), ev_arr)
