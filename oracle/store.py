@@ -58,9 +58,16 @@ Readings where the paper is silent (each also listed in the design doc):
    function needs them): an object put with k > 0 consumers is freed after
    its k-th successful get item; a get frees the objects it brought to zero
    at its end, in the order of the items that brought them there.
+10. Extent placement (``policy = 1``, an alternative to reading 2 that keeps
+    objects contiguous so they can be used in place, §5.3 "pointer
+    rebinding"): the free pages form a set; an object of k pages takes the
+    lowest-numbered run of k consecutive free pages, or, if there is none,
+    the k lowest-numbered free pages. ``free_stack`` then lists the free
+    pages in ascending order (after a compaction too).
 """
 from __future__ import annotations
 
+import bisect
 from dataclasses import dataclass, field
 
 import numpy as np
@@ -104,16 +111,19 @@ class OracleStore:
     writes objects into their pages and reads gets back from the pages (the
     brute-force paged model, for tiny pools)."""
 
-    def __init__(self, pool_bytes: int, page_bytes: int, keep_bytes: bool = True, paged_pool: bool = False):
-        if page_bytes <= 0 or pool_bytes < 0:
-            raise ValueError("bad store geometry")
+    def __init__(self, pool_bytes: int, page_bytes: int, keep_bytes: bool = True, paged_pool: bool = False,
+                 policy: int = 0):
+        if page_bytes <= 0 or pool_bytes < 0 or policy not in (0, 1):
+            raise ValueError("bad store geometry or policy")
+        self.policy = policy
         self.page_bytes = int(page_bytes)
         self.total_pages = int(pool_bytes) // self.page_bytes
         self.limit_pages = self.total_pages
         self.keep_bytes = keep_bytes
         self.pool = np.zeros(self.total_pages * self.page_bytes, np.uint8) if paged_pool else None
-        # free stack: the end of the list is the top; page 0 pops first
-        self.free_stack = list(range(self.total_pages - 1, -1, -1))
+        # reading 2: a stack whose end is the top (page 0 pops first);
+        # reading 10: the free pages in ascending order
+        self.free_stack = list(range(self.total_pages - 1, -1, -1)) if policy == 0 else list(range(self.total_pages))
         self.objects: dict[int, _Object] = {}
         self.evicted: set[int] = set()
         self.next_id = 1
@@ -139,8 +149,28 @@ class OracleStore:
 
     def _release(self, oid: int) -> None:
         for p in self.objects[oid].pages:
-            self.free_stack.append(p)
+            if self.policy == 0:
+                self.free_stack.append(p)
+            else:
+                bisect.insort(self.free_stack, p)
         del self.objects[oid]
+
+    def _take_pages(self, k: int) -> list[int]:
+        if self.policy == 0:
+            return [self.free_stack.pop() for _ in range(k)]
+        if k == 0:
+            return []
+        free = self.free_stack                  # ascending
+        run = None
+        for i in range(len(free) - k + 1):      # the lowest run of k consecutive pages
+            if free[i + k - 1] - free[i] == k - 1:
+                run = free[i:i + k]
+                break
+        if run is None:
+            run = free[:k]                      # else the k lowest pages
+        for p in run:
+            free.remove(p)
+        return run
 
     # -- put ----------------------------------------------------------------
     def _victims(self, demand: int, pinned: set) -> list[int] | None:
@@ -181,7 +211,7 @@ class OracleStore:
         ids = []
         for it in items:
             n = int(it.nbytes)
-            pages = [self.free_stack.pop() for _ in range(pages_for(n, self.page_bytes))]
+            pages = self._take_pages(pages_for(n, self.page_bytes))
             data = None
             if it.data is not None:
                 data = np.ascontiguousarray(it.data).view(np.uint8).reshape(-1).copy()
@@ -297,6 +327,8 @@ class OracleStore:
             moves.append((src, dst, valid))
         own = self.owners()
         self.free_stack = [p for p in range(limit - 1, -1, -1) if p not in own]
+        if self.policy == 1:
+            self.free_stack.reverse()
         self.limit_pages = limit
         self.stats["pages_moved"] += len(moves)
         self.stats["bytes_moved"] += sum(m[2] for m in moves)

@@ -375,3 +375,80 @@ def test_planted_reclaim_before_last_consumer(monkeypatch):
         return st, per, outs
     monkeypatch.setattr(OracleStore, "get_batch", get_batch)
     assert _expect_failure(test_reclaim_by_consumer_count_hand_trace)
+
+
+def test_extent_policy_hand_trace():
+    """Reading 10 (first fit over runs of free pages), worked out by hand
+    (1 KiB pages, 8 pages)."""
+    P = 1024
+    s = OracleStore(8 * P, P, paged_pool=True, policy=1)
+    _, (a,) = s.put_batch([PutItem(3 * P, np.full(3 * P, 1, np.uint8))])
+    _, (b,) = s.put_batch([PutItem(2 * P, np.full(2 * P, 2, np.uint8))])
+    assert s.pages_of(a) == [0, 1, 2] and s.pages_of(b) == [3, 4]
+    assert s.free([a]) == OK and s.free_stack == [0, 1, 2, 5, 6, 7]
+    _, (c,) = s.put_batch([PutItem(4 * P, np.full(4 * P, 3, np.uint8))])
+    assert s.pages_of(c) == [0, 1, 2, 5]       # no run of 4: the 4 lowest pages
+    _, (d,) = s.put_batch([PutItem(P, np.full(P, 4, np.uint8))])
+    assert s.pages_of(d) == [6]
+    assert s.free([b]) == OK and s.free_stack == [3, 4, 7]
+    _, (e,) = s.put_batch([PutItem(2 * P, np.full(2 * P, 5, np.uint8))])
+    assert s.pages_of(e) == [3, 4]             # the run, not the lowest pages 3 and 7
+    assert s.free([c, d, e]) == OK and s.free_stack == list(range(8))
+    _, (x, y, z) = s.put_batch([PutItem(5 * P, None), PutItem(P, None), PutItem(2 * P, None)])
+    assert s.pages_of(x) == [0, 1, 2, 3, 4] and s.pages_of(y) == [5] and s.pages_of(z) == [6, 7]
+    assert s.free([x, z]) == OK                # free runs: 0-4 and 6-7
+    _, (f,) = s.put_batch([PutItem(2 * P, np.full(2 * P, 6, np.uint8))])
+    assert s.pages_of(f) == [0, 1]             # first fit, not best fit (which would take 6, 7)
+    st, moves = s.compact(4 * P)               # live: f = 0, 1 and y = 5 -> y moves to 2
+    assert st == OK and moves == [(5, 2, P)] and s.free_stack == [3]
+
+
+def test_extent_policy_takes_the_lowest_fitting_run():
+    """Brute force: every allocation takes the lowest run of free pages long
+    enough for it, when one exists (runs computed independently here)."""
+    g = np.random.default_rng(3)
+    for seed in range(20):
+        P = 64
+        total = 24
+        s = OracleStore(total * P, P, policy=1)
+        live = []
+        for _ in range(80):
+            if live and g.random() < 0.45:
+                oid = live.pop(int(g.integers(0, len(live))))
+                assert s.free([oid]) == OK
+                continue
+            k = int(g.integers(1, 6))
+            free = sorted(s.free_stack)
+            fits = [free[i] for i in range(len(free) - k + 1) if free[i + k - 1] - free[i] == k - 1]
+            st, ids = s.put_batch([PutItem(k * P, None)])
+            if st != OK:
+                assert len(free) < k
+                continue
+            live.append(ids[0])
+            got = s.pages_of(ids[0])
+            if fits:
+                assert got == list(range(fits[0], fits[0] + k))
+            else:
+                assert got == free[:k]
+            check_invariants(s, {i: None for i in live})
+
+
+def test_planted_best_fit_is_caught(monkeypatch):
+    def take(self, k):
+        if self.policy == 0 or k == 0:
+            return [self.free_stack.pop() for _ in range(k)]
+        free = self.free_stack
+        runs, i = [], 0
+        while i < len(free):
+            j = i
+            while j + 1 < len(free) and free[j + 1] == free[j] + 1:
+                j += 1
+            runs.append((free[i], j - i + 1))
+            i = j + 1
+        ok = sorted([r for r in runs if r[1] >= k], key=lambda r: (r[1], r[0]))
+        run = list(range(ok[0][0], ok[0][0] + k)) if ok else free[:k]
+        for p in run:
+            free.remove(p)
+        return run
+    monkeypatch.setattr(OracleStore, "_take_pages", take)
+    assert _expect_failure(test_extent_policy_hand_trace)
