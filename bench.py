@@ -352,7 +352,8 @@ class WeightRestore:
     per block (layer-wise loading), then got with one get_batch into
     contiguous per-block buffers (each tensor 256-byte aligned in its block)."""
 
-    def __init__(self, device, seed: int = 0, h2d_mode: int = 0, n_blocks: int | None = None):
+    def __init__(self, device, seed: int = 0, h2d_mode: int = 0, n_blocks: int | None = None,
+                 alloc_policy: int = 0):
         import torch
 
         from paper_2607_26566_gb300 import Store, get_descs, put_descs
@@ -366,7 +367,7 @@ class WeightRestore:
             layout = layout[:n_blocks]
         self.specs, self.layout = specs, layout
         self.pool = torch.empty(C_["pool_bytes"], dtype=torch.uint8, device=device)
-        self.store = Store(self.pool, C_["page_bytes"], h2d_mode=h2d_mode)
+        self.store = Store(self.pool, C_["page_bytes"], h2d_mode=h2d_mode, alloc_policy=alloc_policy)
         self.host = []      # pinned per-block source buffers
         self.dst = []       # device per-block destination buffers
         for total, members in layout:
@@ -755,7 +756,8 @@ class PrefixPipeline:
 
         self.torch = torch
         self.device = device
-        self.wr = WeightRestore(device, seed=seed, h2d_mode=1, n_blocks=n_blocks)
+        # extent placement: each tensor lands on consecutive pages, one copy-engine copy per tensor
+        self.wr = WeightRestore(device, seed=seed, h2d_mode=1, n_blocks=n_blocks, alloc_policy=1)
         self.store = self.wr.store
         self.L = len(self.wr.layout)
         self.off = np.zeros(self.L + 1, np.uint32)
@@ -859,7 +861,7 @@ def time_prefix(device, n_blocks: int | None = None, reps: int = 2):
     le_star = prefix_layers_pipeline(pp.t_load, comp)
     mean_load, mean_comp = sum(pp.t_load) / L, sum(comp) / L
     le_eq2 = prefix_layers(L, mean_load, mean_comp)
-    out = {"workload": f"prefix caching: {L}-block DiT weights from pinned host (copy engine), "
+    out = {"workload": f"prefix caching: {L}-block DiT weights from pinned host (copy engine, extent placement), "
                        f"T_load/T_comp = {pp.load_to_comp} per block on average",
            "blocks": L, "t_load_ms_mean": round(mean_load, 4), "t_comp_ms_mean": round(mean_comp, 4),
            "prefix_pipeline": le_star, "prefix_eq2": le_eq2, "compute_only_ms": round(sum(comp), 3), "runs": {}}

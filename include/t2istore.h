@@ -50,6 +50,7 @@ typedef int32_t t2i_status;
 #define T2I_ERR_NOT_FOUND 3 /* id never issued, or already freed                 */
 #define T2I_ERR_EVICTED 4   /* id was evicted to make room (put it again)        */
 #define T2I_ERR_CUDA 5      /* a CUDA call failed; see t2i_last_error            */
+#define T2I_ERR_NOT_CONTIGUOUS 6 /* t2i_view: the object's pages are not consecutive */
 
 /* Object ids: 1, 2, 3, ... in descriptor order, never reused; 0 is never an id. */
 typedef uint64_t t2i_id;
@@ -67,6 +68,12 @@ typedef struct t2i_store_config {
                                 pinned) host memory always takes the copy engine.               */
     uint32_t check_pointers; /* 1 = check every user pointer range with the driver before launch
                                 (recommended); 0 = trust the caller                             */
+    uint32_t alloc_policy;   /* page placement: 0 = LIFO stack of free pages (page 0 first on a
+                                new store; a free pushes pages back in page-list order);
+                                1 = extent: the lowest run of enough consecutive free pages,
+                                else the lowest free pages (objects stay contiguous and can be
+                                used in place, see t2i_view)                                  */
+    uint32_t reserved;       /* must be 0                                                       */
 } t2i_store_config;
 
 /* ---- put ------------------------------------------------------------------
@@ -119,6 +126,7 @@ typedef struct t2i_stats {
     uint64_t launches;   /* kernels launched by the store                                    */
     uint64_t h2d_copies; /* copy-engine copies issued for host sources                        */
     uint64_t reclaimed;  /* objects freed by the store after their last declared consumer    */
+    uint64_t views;      /* successful t2i_view calls                                         */
 } t2i_stats;
 
 typedef struct t2i_object_info {
@@ -181,6 +189,20 @@ t2i_status t2i_get_batch(t2i_store* store, const t2i_get_desc* descs, uint32_t n
 t2i_status t2i_get_batch_after(t2i_store* store, const t2i_get_desc* descs, uint32_t n, t2i_status* per_item,
                                void* cuda_stream, void* wait_event);
 
+/* A zero-copy view of one object (§5.3: the paper wraps arena memory as a
+ * tensor with torch::from_blob and rebinds the model's parameters to it).
+ * If the object's pages are consecutive, *dev_ptr = the device address of
+ * its first byte and *nbytes = its size; else T2I_ERR_NOT_CONTIGUOUS
+ * (alloc_policy 1 keeps objects contiguous whenever a long enough run of
+ * free pages exists). cuda_stream becomes ordered after the call that wrote
+ * the object, so work enqueued on it afterwards may read the bytes in place.
+ * The view stamps recency like a get but counts no consumer. The address is
+ * valid until the object is freed, evicted or moved by a compaction; a later
+ * put that reuses its pages waits for everything enqueued on cuda_stream up
+ * to that put. Reads through the view must not outlive those events.
+ * NOT_FOUND / EVICTED for unknown or evicted ids.                             */
+t2i_status t2i_view(t2i_store* store, t2i_id id, void* cuda_stream, void** dev_ptr, uint64_t* nbytes);
+
 /* Returns the pages of n objects to the free stack (paper §5.3: data is
  * reclaimed when no consumer needs it). Host-only: stream order makes reuse
  * safe. A repeated id is INVALID; an unknown id is NOT_FOUND; in both cases
@@ -214,8 +236,9 @@ const char* t2i_last_error(const t2i_store* store);
  * plans layouts on the host and is what the host-only tests drive.
  * ========================================================================= */
 
-/* total_pages <= 2^32 - 1, page_bytes > 0.                                  */
-t2i_status t2i_ctl_create(uint64_t total_pages, uint64_t page_bytes, t2i_ctl** out);
+/* total_pages <= 2^32 - 1, page_bytes > 0, alloc_policy 0 or 1 (as in
+ * t2i_store_config).                                                         */
+t2i_status t2i_ctl_create(uint64_t total_pages, uint64_t page_bytes, uint32_t alloc_policy, t2i_ctl** out);
 t2i_status t2i_ctl_destroy(t2i_ctl* ctl);
 /* As t2i_put_batch, without copying (src and src_is_host are ignored).      */
 t2i_status t2i_ctl_put(t2i_ctl* ctl, const t2i_put_desc* descs, uint32_t n, t2i_id* out_ids);
@@ -230,7 +253,8 @@ t2i_status t2i_ctl_compact(t2i_ctl* ctl, uint64_t limit_bytes, t2i_move* moves, 
 /* Queries (accept a store's control core). pages receives up to cap page
  * numbers of the object in page-list order; info->n_pages is the full count. */
 t2i_status t2i_ctl_object(const t2i_ctl* ctl, t2i_id id, t2i_object_info* info, uint32_t* pages, uint64_t cap);
-/* The free stack from bottom to top (the top pops first); *n = its size.     */
+/* The free pages: policy 0, the stack from bottom to top (the top pops
+ * first); policy 1, ascending. *n = their number.                            */
 t2i_status t2i_ctl_free_pages(const t2i_ctl* ctl, uint32_t* out, uint64_t cap, uint64_t* n);
 /* Ids evicted by the last put, in eviction order; *n = their number.         */
 t2i_status t2i_ctl_last_evictions(const t2i_ctl* ctl, t2i_id* out, uint64_t cap, uint64_t* n);

@@ -11,13 +11,13 @@ import os
 _HERE = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(_HERE, "libt2istore.so")
 
-OK, ERR_INVALID, ERR_NOSPACE, ERR_NOT_FOUND, ERR_EVICTED, ERR_CUDA = 0, 1, 2, 3, 4, 5
-STATUS_NAMES = {0: "OK", 1: "INVALID", 2: "NOSPACE", 3: "NOT_FOUND", 4: "EVICTED", 5: "CUDA"}
+OK, ERR_INVALID, ERR_NOSPACE, ERR_NOT_FOUND, ERR_EVICTED, ERR_CUDA, ERR_NOT_CONTIGUOUS = 0, 1, 2, 3, 4, 5, 6
+STATUS_NAMES = {0: "OK", 1: "INVALID", 2: "NOSPACE", 3: "NOT_FOUND", 4: "EVICTED", 5: "CUDA", 6: "NOT_CONTIGUOUS"}
 
 
 class StoreConfig(C.Structure):
     _fields_ = [("pool_bytes", C.c_uint64), ("page_bytes", C.c_uint64), ("h2d_mode", C.c_uint32),
-                ("check_pointers", C.c_uint32)]
+                ("check_pointers", C.c_uint32), ("alloc_policy", C.c_uint32), ("reserved", C.c_uint32)]
 
 
 class PutDesc(C.Structure):
@@ -39,7 +39,7 @@ class Stats(C.Structure):
     _fields_ = [(n, C.c_uint64) for n in (
         "total_pages", "limit_pages", "used_pages", "free_pages", "live_objects",
         "bytes_put", "bytes_got", "puts", "gets", "misses", "evictions",
-        "pages_moved", "bytes_moved", "launches", "h2d_copies", "reclaimed")]
+        "pages_moved", "bytes_moved", "launches", "h2d_copies", "reclaimed", "views")]
 
     def as_dict(self) -> dict:
         return {n: int(getattr(self, n)) for n, _ in self._fields_}
@@ -65,12 +65,13 @@ PROTOTYPES = {
     "t2i_put_batch": (_S, [_P, C.POINTER(PutDesc), _U32, _PU64, _P]),
     "t2i_get_batch": (_S, [_P, C.POINTER(GetDesc), _U32, C.POINTER(_S), _P]),
     "t2i_get_batch_after": (_S, [_P, C.POINTER(GetDesc), _U32, C.POINTER(_S), _P, _P]),
+    "t2i_view": (_S, [_P, _U64, _P, C.POINTER(_P), _PU64]),
     "t2i_free": (_S, [_P, _PU64, _U32]),
     "t2i_compact": (_S, [_P, _U64, _P, _PU64]),
     "t2i_store_stats": (_S, [_P, C.POINTER(Stats)]),
     "t2i_store_ctl": (_P, [_P]),
     "t2i_last_error": (C.c_char_p, [_P]),
-    "t2i_ctl_create": (_S, [_U64, _U64, C.POINTER(_P)]),
+    "t2i_ctl_create": (_S, [_U64, _U64, _U32, C.POINTER(_P)]),
     "t2i_ctl_destroy": (_S, [_P]),
     "t2i_ctl_put": (_S, [_P, C.POINTER(PutDesc), _U32, _PU64]),
     "t2i_ctl_get": (_S, [_P, C.POINTER(GetDesc), _U32, C.POINTER(_S)]),

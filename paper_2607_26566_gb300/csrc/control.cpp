@@ -37,12 +37,113 @@ void IdTable::clear(uint64_t id, uint64_t next_id) {
     if (L->used == 0 && (leaf + 1) * kLeafSize <= next_id) leaves_[leaf].reset();
 }
 
-// ---------------------------------------------------------------- Control
-Control::Control(uint64_t total_pages, uint64_t page_bytes)
-    : P_(page_bytes), total_pages_(total_pages), limit_pages_(total_pages) {
-    free_.reserve(total_pages);
-    for (uint64_t p = total_pages; p-- > 0;) free_.push_back(static_cast<uint32_t>(p));
+// ---------------------------------------------------------------- FreePages
+FreePages::FreePages(uint64_t total_pages, uint32_t policy) : policy_(policy), count_(total_pages) {
+    if (policy_ == 0) {
+        stack_.reserve(total_pages);
+        for (uint64_t p = total_pages; p-- > 0;) stack_.push_back(static_cast<uint32_t>(p));
+    } else if (total_pages) {
+        runs_[0] = static_cast<uint32_t>(total_pages);
+    }
 }
+
+void FreePages::take(uint64_t k, std::vector<uint32_t>* out) {
+    out->resize(k);
+    count_ -= k;
+    if (policy_ == 0) {
+        for (uint64_t j = 0; j < k; ++j) {
+            (*out)[j] = stack_.back();
+            stack_.pop_back();
+        }
+        return;
+    }
+    if (k == 0) return;
+    for (auto it = runs_.begin(); it != runs_.end(); ++it) {  // first fit
+        if (it->second >= k) {
+            const uint32_t start = it->first, len = it->second;
+            runs_.erase(it);
+            if (len > k) runs_[start + uint32_t(k)] = len - uint32_t(k);
+            for (uint64_t j = 0; j < k; ++j) (*out)[j] = start + uint32_t(j);
+            return;
+        }
+    }
+    uint64_t j = 0;  // no run is long enough: the lowest pages
+    while (j < k) {
+        auto it = runs_.begin();
+        const uint32_t start = it->first, len = it->second;
+        const uint32_t m = uint32_t(std::min<uint64_t>(len, k - j));
+        runs_.erase(it);
+        if (len > m) runs_[start + m] = len - m;
+        for (uint32_t t = 0; t < m; ++t) (*out)[j++] = start + t;
+    }
+}
+
+void FreePages::insert_page(uint32_t p) {
+    auto next = runs_.lower_bound(p);
+    if (next != runs_.begin()) {
+        auto prev = std::prev(next);
+        if (prev->first + prev->second == p) {
+            prev->second++;
+            if (next != runs_.end() && next->first == p + 1) {
+                prev->second += next->second;
+                runs_.erase(next);
+            }
+            return;
+        }
+    }
+    if (next != runs_.end() && next->first == p + 1) {
+        const uint32_t len = next->second + 1;
+        runs_.erase(next);
+        runs_[p] = len;
+    } else {
+        runs_[p] = 1;
+    }
+}
+
+void FreePages::give(const std::vector<uint32_t>& pages) {
+    count_ += pages.size();
+    if (policy_ == 0) {
+        for (uint32_t p : pages) stack_.push_back(p);
+        return;
+    }
+    for (uint32_t p : pages) insert_page(p);
+}
+
+void FreePages::rebuild(uint64_t limit, const std::vector<uint8_t>& used) {
+    stack_.clear();
+    runs_.clear();
+    count_ = 0;
+    if (policy_ == 0) {
+        for (uint64_t p = limit; p-- > 0;)
+            if (!used[p]) stack_.push_back(static_cast<uint32_t>(p));
+        count_ = stack_.size();
+        return;
+    }
+    uint64_t p = 0;
+    while (p < limit) {
+        if (used[p]) {
+            ++p;
+            continue;
+        }
+        const uint64_t start = p;
+        while (p < limit && !used[p]) ++p;
+        runs_[uint32_t(start)] = uint32_t(p - start);
+        count_ += p - start;
+    }
+}
+
+std::vector<uint32_t> FreePages::list() const {
+    if (policy_ == 0) return stack_;
+    std::vector<uint32_t> out;
+    out.reserve(count_);
+    for (const auto& r : runs_)
+        for (uint32_t t = 0; t < r.second; ++t) out.push_back(r.first + t);
+    return out;
+}
+
+// ---------------------------------------------------------------- Control
+Control::Control(uint64_t total_pages, uint64_t page_bytes, uint32_t policy)
+    : P_(page_bytes), total_pages_(total_pages), limit_pages_(total_pages), free_(total_pages, policy) {}
 
 Control::~Control() {
     for (Object* o : live_) delete o;
@@ -84,7 +185,7 @@ void Control::flush_touches() {
 
 void Control::release(Object* o, bool evicted) {
     const uint64_t np = o->pages.size();
-    for (uint32_t p : o->pages) free_.push_back(p);
+    free_.give(o->pages);
     used_pages_ -= np;
     Group* g = o->group;
     g->n_objects--;
@@ -114,6 +215,31 @@ uint64_t Control::live_pages_at_or_above(uint64_t limit) const {
     for (const Object* o : live_)
         for (uint32_t p : o->pages) k += p >= limit;
     return k;
+}
+
+t2i_status Control::view(uint64_t id, const Object** out) {
+    *out = nullptr;
+    const uintptr_t v = ids_.get(id);
+    if (v == 0) {
+        err_ = "view: id " + std::to_string(id) + " not found";
+        return T2I_ERR_NOT_FOUND;
+    }
+    if (v == IdTable::kEvicted) {
+        err_ = "view: id " + std::to_string(id) + " was evicted";
+        return T2I_ERR_EVICTED;
+    }
+    Object* o = reinterpret_cast<Object*>(v);
+    for (size_t j = 1; j < o->pages.size(); ++j) {
+        if (o->pages[j] != o->pages[0] + j) {
+            err_ = "view: the object's pages are not consecutive";
+            return T2I_ERR_NOT_CONTIGUOUS;
+        }
+    }
+    touch(o);
+    flush_touches();
+    counters_.views++;
+    *out = o;
+    return T2I_OK;
 }
 
 const Object* Control::find(uint64_t id) const {
@@ -190,11 +316,7 @@ t2i_status Control::put(const t2i_put_desc* descs, uint32_t n, t2i_id* ids, std:
         o->consumers_left = d.consumers;
         o->group = group_for(d.group);
         const uint64_t np = pages_for(d.nbytes);
-        o->pages.resize(np);
-        for (uint64_t j = 0; j < np; ++j) {
-            o->pages[j] = free_.back();
-            free_.pop_back();
-        }
+        free_.take(np, &o->pages);
         used_pages_ += np;
         Group* g = o->group;
         g->n_objects++;
@@ -354,9 +476,7 @@ t2i_status Control::compact(uint64_t limit_bytes, std::vector<t2i_move>* moves) 
         moves->push_back({t.page, dst, valid});
         moved_bytes += valid;
     }
-    free_.clear();
-    for (uint64_t p = limit; p-- > 0;)
-        if (!used[p]) free_.push_back(static_cast<uint32_t>(p));
+    free_.rebuild(limit, used);
     limit_pages_ = limit;
     counters_.pages_moved += tail.size();
     counters_.bytes_moved += moved_bytes;

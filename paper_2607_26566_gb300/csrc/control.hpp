@@ -8,9 +8,14 @@
 // directory id -> {size, tags, page list}. Eviction follows §5.3: least
 // recently used model first, its layers in reverse order, until the demand is
 // met. Where the paper is silent the rules are:
-//   - free pages form a LIFO stack; page 0 pops first on a new store; a put
-//     pops its pages one at a time, objects in descriptor order; a free pushes
-//     an object's pages back in page-list order;
+//   - placement policy 0 (LIFO): free pages form a stack; page 0 pops first
+//     on a new store; a put pops its pages one at a time, objects in
+//     descriptor order; a free pushes an object's pages back in page-list
+//     order;
+//   - placement policy 1 (extent): free pages form a set of runs; an object
+//     of k pages takes the lowest-numbered run of k consecutive free pages,
+//     else the k lowest-numbered free pages (objects stay contiguous, so they
+//     can be used in place);
 //   - ids are 1, 2, 3, ... in descriptor order and never reused;
 //   - recency is per group, stamped once per object put or got, in
 //     descriptor order; victims: least recent group first, then the highest
@@ -26,6 +31,7 @@
 #pragma once
 
 #include <cstdint>
+#include <map>
 #include <memory>
 #include <set>
 #include <string>
@@ -62,6 +68,29 @@ struct Group {
     std::set<std::pair<uint32_t, uint64_t>, std::greater<std::pair<uint32_t, uint64_t>>> victims;
 };
 
+// The free pages under either placement policy.
+class FreePages {
+  public:
+    FreePages(uint64_t total_pages, uint32_t policy);
+    uint64_t size() const { return count_; }
+    uint32_t policy() const { return policy_; }
+    // k pages for one object, in page-list order (requires k <= size())
+    void take(uint64_t k, std::vector<uint32_t>* out);
+    // an object's pages back, in page-list order
+    void give(const std::vector<uint32_t>& pages);
+    // after a compaction: every page below limit that `used` does not mark
+    void rebuild(uint64_t limit, const std::vector<uint8_t>& used);
+    // policy 0: the stack from bottom to top; policy 1: ascending
+    std::vector<uint32_t> list() const;
+
+  private:
+    void insert_page(uint32_t p);
+    uint32_t policy_;
+    uint64_t count_ = 0;
+    std::vector<uint32_t> stack_;          // policy 0; back() is the top
+    std::map<uint32_t, uint32_t> runs_;    // policy 1: first page -> run length
+};
+
 // id -> object, or the "evicted" tombstone; two-level table over the dense
 // id space whose leaves are released once every id in them is gone.
 class IdTable {
@@ -84,7 +113,7 @@ class IdTable {
 
 class Control {
   public:
-    Control(uint64_t total_pages, uint64_t page_bytes);
+    Control(uint64_t total_pages, uint64_t page_bytes, uint32_t policy = 0);
     ~Control();
     Control(const Control&) = delete;
     Control& operator=(const Control&) = delete;
@@ -115,7 +144,11 @@ class Control {
     uint64_t live_pages_at_or_above(uint64_t limit) const;
     const Object* find(uint64_t id) const;
     bool is_evicted(uint64_t id) const { return ids_.get(id) == IdTable::kEvicted; }
-    const std::vector<uint32_t>& free_stack() const { return free_; }
+    std::vector<uint32_t> free_list() const { return free_.list(); }
+    // A view: the object's first page if its pages are consecutive (stamps
+    // recency like a get, counts no consumer). NOT_FOUND / EVICTED /
+    // NOT_CONTIGUOUS otherwise.
+    t2i_status view(uint64_t id, const Object** out);
     const std::vector<t2i_id>& last_evictions() const { return last_evictions_; }
     void stats(t2i_stats* out) const;
     t2i_stats& counters() { return counters_; }
@@ -138,7 +171,7 @@ class Control {
     uint64_t next_id_ = 1;
     uint64_t clock_ = 0;
     uint64_t epoch_ = 1;            // groups start at epoch 0, so the first batch is new
-    std::vector<uint32_t> free_;   // free page stack; back() is the top
+    FreePages free_;
     IdTable ids_;
     std::vector<Object*> live_;
     std::unordered_map<uint64_t, std::unique_ptr<Group>> groups_;

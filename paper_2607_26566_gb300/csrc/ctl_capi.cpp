@@ -25,18 +25,18 @@ using t2i::Control;
 
 extern "C" {
 
-t2i_status t2i_ctl_create(uint64_t total_pages, uint64_t page_bytes, t2i_ctl** out) {
+t2i_status t2i_ctl_create(uint64_t total_pages, uint64_t page_bytes, uint32_t alloc_policy, t2i_ctl** out) {
     if (!out) {
         t2i::set_thread_error("t2i_ctl_create: null out");
         return T2I_ERR_INVALID;
     }
     *out = nullptr;
-    if (page_bytes == 0 || total_pages > 0xFFFFFFFFull) {
-        t2i::set_thread_error("t2i_ctl_create: page_bytes must be > 0 and total_pages < 2^32");
+    if (page_bytes == 0 || total_pages > 0xFFFFFFFFull || alloc_policy > 1) {
+        t2i::set_thread_error("t2i_ctl_create: page_bytes must be > 0, total_pages < 2^32, alloc_policy 0 or 1");
         return T2I_ERR_INVALID;
     }
     try {
-        t2i_ctl* c = new t2i_ctl{new Control(total_pages, page_bytes), true};
+        t2i_ctl* c = new t2i_ctl{new Control(total_pages, page_bytes, alloc_policy), true};
         *out = c;
     } catch (const std::bad_alloc&) {
         t2i::set_thread_error("t2i_ctl_create: host memory allocation failed");
@@ -121,7 +121,7 @@ t2i_status t2i_ctl_object(const t2i_ctl* ctl, t2i_id id, t2i_object_info* info, 
 
 t2i_status t2i_ctl_free_pages(const t2i_ctl* ctl, uint32_t* out, uint64_t cap, uint64_t* n) {
     if (!ctl) return T2I_ERR_INVALID;
-    const auto& f = ctl->core->free_stack();
+    const std::vector<uint32_t> f = ctl->core->free_list();
     if (n) *n = f.size();
     if (out) {
         const uint64_t k = f.size() < cap ? f.size() : cap;

@@ -36,6 +36,9 @@ class StreamDeps {
         uint8_t more_readers = 0;  // > 2 reading streams since the last write
     };
     static constexpr uint32_t kRing = 64;
+    // a reader whose reads are not calls of the store (a view): later
+    // writers wait for everything its stream has been given by then
+    static constexpr uint32_t kOpen = 0xFFFFFFFFu;
 
     ~StreamDeps() { release(); }
 

@@ -102,7 +102,7 @@ class Store {
   public:
     Store(void* pool, const t2i_store_config& cfg, int device)
         : pool_(reinterpret_cast<uint64_t>(pool)), cfg_(cfg), device_(device),
-          ctl_(cfg.pool_bytes / cfg.page_bytes, cfg.page_bytes) {
+          ctl_(cfg.pool_bytes / cfg.page_bytes, cfg.page_bytes, cfg.alloc_policy) {
         handle_.core = &ctl_;
         handle_.owned = false;
         page_shift_ = log2_exact(cfg.page_bytes);
@@ -153,6 +153,7 @@ class Store {
         return st;
     }
     t2i_status compact(uint64_t limit_bytes, cudaStream_t stream, uint64_t* moved);
+    t2i_status view(t2i_id id, cudaStream_t stream, void** ptr, uint64_t* nbytes);
 
   private:
     // ---- pointer checks (per call cache of the last allocation seen)
@@ -575,6 +576,33 @@ t2i_status Store::get(const t2i_get_desc* descs, uint32_t n, t2i_status* per_ite
     return st;
 }
 
+t2i_status Store::view(t2i_id id, cudaStream_t stream, void** ptr, uint64_t* nbytes) {
+    if (!ptr) {
+        err_ = "view: null output";
+        return T2I_ERR_INVALID;
+    }
+    *ptr = nullptr;
+    if (nbytes) *nbytes = 0;
+    const Object* o = nullptr;
+    t2i_status st = ctl_.view(id, &o);
+    if (st != T2I_OK) {
+        err_ = ctl_.error();
+        return st;
+    }
+    if (nbytes) *nbytes = o->nbytes;
+    if (o->pages.empty()) return T2I_OK;
+    DeviceGuard g(device_);
+    int si = 0;
+    if ((st = stream_slot(stream, &si)) != T2I_OK) return st;
+    deps_.begin(si);
+    for (uint32_t pg : o->pages) deps_.reads(pg);
+    cudaError_t we = deps_.wait();
+    if (we != cudaSuccess) return cuda_fail("view: cannot order after the object's writer", we);
+    for (uint32_t pg : o->pages) deps_.mark_read(pg, StreamDeps::kOpen);
+    *ptr = reinterpret_cast<void*>(pool_ + (uint64_t(o->pages[0]) << page_shift_));
+    return T2I_OK;
+}
+
 t2i_status Store::compact(uint64_t limit_bytes, cudaStream_t stream, uint64_t* moved) {
     std::vector<t2i_move> moves;
     t2i_status st = ctl_.compact(limit_bytes, &moves);
@@ -636,7 +664,8 @@ t2i_status t2i_store_create(void* pool_dev, const t2i_store_config* cfg, int dev
         t2i::set_thread_error("t2i_store_create: page_bytes must be a power of two in [256 B, 1 GiB]");
         return T2I_ERR_INVALID;
     }
-    if (cfg->pool_bytes / cfg->page_bytes > 0xFFFFFFFFull || cfg->h2d_mode > 1 || cfg->check_pointers > 1) {
+    if (cfg->pool_bytes / cfg->page_bytes > 0xFFFFFFFFull || cfg->h2d_mode > 1 || cfg->check_pointers > 1 ||
+        cfg->alloc_policy > 1 || cfg->reserved != 0) {
         t2i::set_thread_error("t2i_store_create: too many pages or a bad flag");
         return T2I_ERR_INVALID;
     }
@@ -746,6 +775,10 @@ t2i_status t2i_put_layers(t2i_store* store, const t2i_put_desc* descs, const uin
         }
     }
     return T2I_OK;
+}
+
+t2i_status t2i_view(t2i_store* store, t2i_id id, void* cuda_stream, void** dev_ptr, uint64_t* nbytes) {
+    T2I_STORE_CALL(store, store->s->view(id, static_cast<cudaStream_t>(cuda_stream), dev_ptr, nbytes));
 }
 
 t2i_status t2i_compact(t2i_store* store, uint64_t limit_bytes, void* cuda_stream, uint64_t* pages_moved) {

@@ -105,7 +105,8 @@ class Ctl:
     """The host control core alone (t2i_ctl_*): page allocator, directory,
     LRU and compaction planner without device memory."""
 
-    def __init__(self, total_pages: int = 0, page_bytes: int = 0, _borrowed=None, _owner=None):
+    def __init__(self, total_pages: int = 0, page_bytes: int = 0, alloc_policy: int = 0, _borrowed=None,
+                 _owner=None):
         self._lib = L.load()
         self._owner = _owner
         if _borrowed is not None:
@@ -113,7 +114,7 @@ class Ctl:
             self._owned = False
             return
         h = C.c_void_p()
-        st = self._lib.t2i_ctl_create(total_pages, page_bytes, C.byref(h))
+        st = self._lib.t2i_ctl_create(total_pages, page_bytes, alloc_policy, C.byref(h))
         if st != L.OK:
             raise T2IError(st, self._lib.t2i_ctl_last_error(None).decode())
         self._h = h
@@ -194,7 +195,7 @@ class Store:
     tensor (kept alive by the store object) or an address with ``pool_bytes``."""
 
     def __init__(self, pool, page_bytes: int, pool_bytes: int | None = None, device: int | None = None,
-                 h2d_mode: int = 0, check_pointers: int = 1):
+                 h2d_mode: int = 0, check_pointers: int = 1, alloc_policy: int = 0):
         self._lib = L.load()
         self.pool = pool
         if pool_bytes is None:
@@ -204,7 +205,7 @@ class Store:
         self.device = device
         self.page_bytes = int(page_bytes)
         self.pool_bytes = int(pool_bytes)
-        cfg = L.StoreConfig(pool_bytes, page_bytes, h2d_mode, check_pointers)
+        cfg = L.StoreConfig(pool_bytes, page_bytes, h2d_mode, check_pointers, alloc_policy, 0)
         h = C.c_void_p()
         st = self._lib.t2i_store_create(C.c_void_p(_ptr(pool)), C.byref(cfg), device, C.byref(h))
         if st != L.OK:
@@ -248,6 +249,27 @@ class Store:
     def free(self, ids) -> int:
         ids = np.ascontiguousarray(ids, np.uint64)
         return self._lib.t2i_free(self._h, ids.ctypes.data_as(C.POINTER(C.c_uint64)), len(ids))
+
+    def view(self, oid: int, stream=None):
+        """(status, device address, nbytes) -- t2i_view."""
+        ptr = C.c_void_p()
+        n = C.c_uint64()
+        st = self._lib.t2i_view(self._h, oid, _stream(stream), C.byref(ptr), C.byref(n))
+        return st, int(ptr.value or 0), int(n.value)
+
+    def tensor_view(self, oid: int, dtype=None, shape=None, stream=None):
+        """The object as a tensor over the pool, without a copy (the pool must
+        be a torch tensor): status, tensor (None on failure)."""
+        st, ptr, n = self.view(oid, stream)
+        if st != L.OK:
+            return st, None
+        off = ptr - int(self.pool.data_ptr()) if n else 0
+        t = self.pool.view(-1)[off:off + n]
+        if dtype is not None:
+            t = t.view(dtype)
+        if shape is not None:
+            t = t.view(shape)
+        return st, t
 
     def put_layers(self, descs: np.ndarray, layer_off, first: int = 0, stream=None, events=None):
         """(status, ids) -- t2i_put_layers. ``layer_off``: n_layers + 1 offsets

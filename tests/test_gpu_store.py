@@ -496,3 +496,50 @@ def test_cross_stream_compaction():
     assert st.get_batch(get_descs([int(ia)], [out]), stream=s3)[0] == 0
     torch.cuda.synchronize()
     assert torch.equal(out, a)
+
+
+def test_views_in_place():
+    """Extent placement keeps objects contiguous; a view reads them in place
+    (no copy) and equals what was put."""
+    P = 64 * 1024
+    st = make_store(64 * P, P, alloc_policy=1)
+    xs = [torch.randint(0, 256, (n,), dtype=torch.uint8, device=DEV) for n in (3 * P + 5, P, 10, 7 * P)]
+    s, ids = st.put_batch(put_descs(xs))
+    assert s == 0
+    for i, x in zip(ids, xs):
+        s, t = st.tensor_view(int(i))
+        assert s == 0 and t.data_ptr() != x.data_ptr() and torch.equal(t, x)
+    assert st.stats()["views"] == len(xs)
+    # LIFO placement after a free hands pages out in descending order: no view
+    st0 = make_store(8 * P, P)
+    a = torch.randint(0, 256, (2 * P,), dtype=torch.uint8, device=DEV)
+    s, (ia, ib) = st0.put_batch(put_descs([a, a]))
+    assert st0.free([int(ia)]) == 0
+    s, (ic,) = st0.put_batch(put_descs([a]))
+    assert st0.ctl.object(int(ic))[2] == [1, 0]
+    assert st0.view(int(ic))[0] == 6                       # NOT_CONTIGUOUS
+    assert st0.view(int(ib))[0] == 0 and st0.view(999)[0] == 3
+
+
+def test_view_is_ordered_after_its_writer_and_before_reuse():
+    """A view on one stream waits for a late put on another; a put reusing
+    the viewed pages waits for the view stream's late reads."""
+    P = 64 * 1024
+    st = make_store(8 * P, P, alloc_policy=1)
+    s1, s2, s3 = torch.cuda.Stream(), torch.cuda.Stream(), torch.cuda.Stream()
+    x = torch.randint(0, 256, (8 * P,), dtype=torch.uint8, device=DEV)
+    y = torch.randint(0, 256, (8 * P,), dtype=torch.uint8, device=DEV)
+    torch.cuda.synchronize()
+    _late(s1, 30)
+    s, (ix,) = st.put_batch(put_descs([x]), stream=s1)
+    assert s == 0
+    s, t = st.tensor_view(int(ix), stream=s2)
+    assert s == 0
+    _late(s2, 30)
+    with torch.cuda.stream(s2):
+        z = t.clone()                         # a late reader, in place
+    assert st.free([int(ix)]) == 0
+    s, (iy,) = st.put_batch(put_descs([y]), stream=s3)   # the same pages
+    assert s == 0 and st.ctl.object(int(iy))[2] == list(range(8))
+    torch.cuda.synchronize()
+    assert torch.equal(z, x)
