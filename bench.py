@@ -55,7 +55,7 @@ def parse():
     p.add_argument("--sweep", action="store_true", help="also time B = 1 and B = 4")
     p.add_argument("--pool-gib", type=float, default=None, help="smaller pool (profiling small cases)")
     p.add_argument("--cpu-seconds", type=float, default=10.0, help="minimum CPU-baseline sample time")
-    p.add_argument("--rows", default="weights,adapters,compaction,prefix",
+    p.add_argument("--rows", default="weights,adapters,compaction,prefix,views",
                    help="other hot-path rows timed in the same run (comma list, or 'none')")
     p.add_argument("--adapter-calls", type=int, default=10_000)
     p.add_argument("--rows-only", action="store_true", help="skip the handoff headline (profiling a row)")
@@ -880,6 +880,64 @@ def time_prefix(device, n_blocks: int | None = None, reps: int = 2):
     return out
 
 
+# ----------------------------------------------------------------------------- views
+def contiguous_fraction(store, ids) -> tuple[float, int]:
+    """Fraction of the live multi-page objects among ``ids`` whose pages are
+    consecutive (those a view can serve), and how many were looked at."""
+    n = ok = 0
+    for i in ids:
+        st, info, pages = store.ctl.object(int(i))
+        if st != 0 or len(pages) < 2:
+            continue
+        n += 1
+        ok += all(pages[j] == pages[0] + j for j in range(len(pages)))
+    return (ok / n if n else 1.0), n
+
+
+def time_views(device, adapter_calls: int = 3000):
+    """Zero-copy views: the weight restore with extent placement (every tensor
+    viewed in place instead of copied out), and how contiguous the adapter
+    cache stays under each placement policy after eviction churn."""
+    import torch
+
+    out = {"workload": "views: weight restore (extent placement) and adapter-cache contiguity per policy"}
+    wr = WeightRestore(device, alloc_policy=1)
+    wr.put_all()
+    torch.cuda.synchronize(device)
+    t = time.perf_counter()
+    ok = 0
+    for i in wr.ids:
+        ok += wr.store.view(int(i))[0] == 0
+    dt = time.perf_counter() - t
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record()
+    wr.get_all()
+    e1.record()
+    torch.cuda.synchronize(device)
+    out["weights_viewable"] = f"{ok}/{len(wr.ids)}"
+    out["weights_view_host_us"] = round(1e6 * dt / len(wr.ids), 2)
+    out["weights_all_views_ms"] = round(1e3 * dt, 3)
+    out["weights_copy_get_ms"] = round(e0.elapsed_time(e1), 3)
+    wr.close()
+    del wr
+    torch.cuda.empty_cache()
+    for policy in (0, 1):
+        ad = Adapters(device, n_calls=adapter_calls)
+        ad.store.close()
+        from paper_2607_26566_gb300 import Store
+        ad.store = Store(ad.pool, W.ADAPTERS["page_bytes"], alloc_policy=policy)
+        for k in range(adapter_calls):
+            ad.call(k)
+        ids = [i for v in ad.ids.values() for i in v]
+        frac, n = contiguous_fraction(ad.store, ids)
+        out[f"adapters_policy{policy}_contiguous"] = round(frac, 4)
+        out[f"adapters_policy{policy}_multipage_objects"] = n
+        ad.close()
+        del ad
+        torch.cuda.empty_cache()
+    return out
+
+
 # ----------------------------------------------------------------------------- CPU (oracle)
 def oracle_sample(B: int, n_requests: int, min_seconds: float = 0.0, max_steps: int = 1):
     """The oracle as it stands on the host: steps of the handoff workload (put
@@ -958,6 +1016,8 @@ def run_rows(args, device, peak):
         rows["compaction"] = time_compaction(device, pool_gib=args.compaction_gib)
     if "prefix" in wanted:
         rows["prefix"] = time_prefix(device)
+    if "views" in wanted:
+        rows["views"] = time_views(device)
     for r in rows.values():
         for k in ("get_gbs", "gbs", "hit_gbs"):
             if k in r:
