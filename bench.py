@@ -55,7 +55,7 @@ def parse():
     p.add_argument("--sweep", action="store_true", help="also time B = 1 and B = 4")
     p.add_argument("--pool-gib", type=float, default=None, help="smaller pool (profiling small cases)")
     p.add_argument("--cpu-seconds", type=float, default=10.0, help="minimum CPU-baseline sample time")
-    p.add_argument("--rows", default="weights,adapters,compaction,prefix,views",
+    p.add_argument("--rows", default="weights,adapters,compaction,prefix,views,pull",
                    help="other hot-path rows timed in the same run (comma list, or 'none')")
     p.add_argument("--adapter-calls", type=int, default=10_000)
     p.add_argument("--rows-only", action="store_true", help="skip the handoff headline (profiling a row)")
@@ -938,6 +938,59 @@ def time_views(device, adapter_calls: int = 3000):
     return out
 
 
+# ----------------------------------------------------------------------------- pull
+def time_pull(device, B: int = 8, requests: int = 64, reps: int = 3):
+    """Producer -> consumer store pulls (§5.2) of the handoff intermediates:
+    one t2i_pull per request, page to page, then the consumer frees them."""
+    import torch
+
+    from paper_2607_26566_gb300 import Store
+
+    hw = Handoff(B, requests, device)
+    stream = torch.cuda.current_stream(device)
+    cons_pool = torch.empty(W.HANDOFF["pool_bytes"], dtype=torch.uint8, device=device)
+    cons = Store(cons_pool, W.HANDOFF["page_bytes"])
+    n = hw.n_obj
+    for r in range(requests):     # the producers' outputs
+        st, ids = hw.store.put_batch(hw.pd[r])
+        hw.store.check(st)
+        hw.ids[n * r:n * (r + 1)] = ids
+    payload = sum(sp.nbytes for sp in hw.specs) * requests
+
+    def once():
+        new = []
+        for r in range(requests):
+            st, out, _ = cons.pull(hw.store, hw.ids[n * r:n * (r + 1)])
+            cons.check(st)
+            new.append(out)
+        cons.check(cons.free(np.concatenate(new)))
+
+    once()
+    torch.cuda.synchronize(device)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(reps):
+        once()
+    e1.record(stream)
+    torch.cuda.synchronize(device)
+    ms = e0.elapsed_time(e1) / reps
+    # the consumer's bytes equal the producer's (a sample request)
+    from paper_2607_26566_gb300 import get_descs
+    st, out, _ = cons.pull(hw.store, hw.ids[:n])
+    cons.check(st)
+    dst = [torch.empty(sp.nbytes, dtype=torch.uint8, device=device) for sp in hw.specs]
+    cons.check(cons.get_batch(get_descs(out, dst), per_item=False)[0])
+    torch.cuda.synchronize(device)
+    ok = all(torch.equal(t.reshape(-1).view(torch.uint8), d) for t, d in zip(hw.inputs[0], dst))
+    res = {"workload": f"pull: {requests} handoff requests (B={B}) from a producer store into a consumer store",
+           "ms": round(ms, 3), "gbs": round(2 * payload / (ms * 1e-3) / 1e9, 1), "bit_exact": bool(ok)}
+    cons.close()
+    hw.store.close()
+    del hw, cons, cons_pool
+    torch.cuda.empty_cache()
+    return res
+
+
 # ----------------------------------------------------------------------------- CPU (oracle)
 def oracle_sample(B: int, n_requests: int, min_seconds: float = 0.0, max_steps: int = 1):
     """The oracle as it stands on the host: steps of the handoff workload (put
@@ -1018,6 +1071,8 @@ def run_rows(args, device, peak):
         rows["prefix"] = time_prefix(device)
     if "views" in wanted:
         rows["views"] = time_views(device)
+    if "pull" in wanted:
+        rows["pull"] = time_pull(device)
     for r in rows.values():
         for k in ("get_gbs", "gbs", "hit_gbs"):
             if k in r:

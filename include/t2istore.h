@@ -203,6 +203,21 @@ t2i_status t2i_get_batch_after(t2i_store* store, const t2i_get_desc* descs, uint
  * NOT_FOUND / EVICTED for unknown or evicted ids.                             */
 t2i_status t2i_view(t2i_store* store, t2i_id id, void* cuda_stream, void** dev_ptr, uint64_t* nbytes);
 
+/* Pulls n objects of the producer's store `src` into the consumer's store
+ * `dst` (§5.2: the consumer allocates a block in its own arena and pulls the
+ * producer's bytes into it), page to page on the GPU, without a staging
+ * buffer. out_ids[i] receives the new id in dst of src_ids[i]; the new
+ * objects are intermediates (evictable = 0, group 0, order 0) with the
+ * source's dtype_tag and `consumers`. The sources are read like a get
+ * (recency stamped, one consumer counted). Every source id is checked first
+ * (per_item, nullable: OK / NOT_FOUND / EVICTED); NOSPACE in dst changes
+ * nothing. Both stores must be distinct, on the same device and have the
+ * same page size (INVALID otherwise). The copy is ordered after the
+ * producer's write of the source pages and after the consumer store's
+ * earlier users of the new pages.                                            */
+t2i_status t2i_pull(t2i_store* dst, t2i_store* src, const t2i_id* src_ids, uint32_t n, uint32_t consumers,
+                    t2i_id* out_ids, t2i_status* per_item, void* cuda_stream);
+
 /* Returns the pages of n objects to the free stack (paper §5.3: data is
  * reclaimed when no consumer needs it). Host-only: stream order makes reuse
  * safe. A repeated id is INVALID; an unknown id is NOT_FOUND; in both cases

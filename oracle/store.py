@@ -64,6 +64,7 @@ Readings where the paper is silent (each also listed in the design doc):
     lowest-numbered run of k consecutive free pages, or, if there is none,
     the k lowest-numbered free pages. ``free_stack`` then lists the free
     pages in ascending order (after a compaction too).
+11. Pull between stores (§5.2): see :meth:`OracleStore.pull`.
 """
 from __future__ import annotations
 
@@ -277,6 +278,36 @@ class OracleStore:
             self._release(oid)
             self.stats["reclaimed"] += 1
         return OK, per, outs
+
+    # -- pull (§5.2) ----------------------------------------------------------
+    def pull(self, src: "OracleStore", ids, consumers: int = 0):
+        """The consumer (self) allocates room in its own store and pulls the
+        producer's (src) objects into it (§5.2). Reading 11: every id is
+        checked first (statuses as a get's); the new objects are put like
+        intermediates (evictable = 0, group 0, order 0, the source's dtype
+        tag, ``consumers``); if they do not fit, NOSPACE and nothing happens;
+        otherwise the sources are read like a get (recency stamped, one
+        consumer counted). Returns (status, per-item statuses, new ids)."""
+        if self.page_bytes != src.page_bytes:
+            return INVALID, [], []
+        per = []
+        for oid in ids:
+            oid = int(oid)
+            per.append(OK if oid in src.objects else EVICTED if oid in src.evicted else NOT_FOUND)
+        bad = [x for x in per if x != OK]
+        if bad:
+            src.stats["misses"] += sum(1 for x in per if x == EVICTED)
+            return bad[0], per, []
+        items = []
+        for oid in ids:
+            o = src.objects[int(oid)]
+            data = src._read(o)
+            items.append(PutItem(o.nbytes, data, o.dtype_tag, 0, 0, False, int(consumers)))
+        st, new_ids = self.put_batch(items)
+        if st != OK:
+            return st, per, []
+        src.get_batch(ids)
+        return OK, per, new_ids
 
     # -- free ---------------------------------------------------------------
     def free(self, ids) -> int:

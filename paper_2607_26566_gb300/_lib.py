@@ -66,6 +66,7 @@ PROTOTYPES = {
     "t2i_get_batch": (_S, [_P, C.POINTER(GetDesc), _U32, C.POINTER(_S), _P]),
     "t2i_get_batch_after": (_S, [_P, C.POINTER(GetDesc), _U32, C.POINTER(_S), _P, _P]),
     "t2i_view": (_S, [_P, _U64, _P, C.POINTER(_P), _PU64]),
+    "t2i_pull": (_S, [_P, _P, _PU64, _U32, _U32, _PU64, C.POINTER(_S), _P]),
     "t2i_free": (_S, [_P, _PU64, _U32]),
     "t2i_compact": (_S, [_P, _U64, _P, _PU64]),
     "t2i_store_stats": (_S, [_P, C.POINTER(Stats)]),

@@ -154,6 +154,8 @@ class Store {
     }
     t2i_status compact(uint64_t limit_bytes, cudaStream_t stream, uint64_t* moved);
     t2i_status view(t2i_id id, cudaStream_t stream, void** ptr, uint64_t* nbytes);
+    t2i_status pull_from(Store& src, const t2i_id* ids, uint32_t n, uint32_t consumers, t2i_id* out_ids,
+                         t2i_status* per_item, cudaStream_t stream);
 
   private:
     // ---- pointer checks (per call cache of the last allocation seen)
@@ -603,6 +605,96 @@ t2i_status Store::view(t2i_id id, cudaStream_t stream, void** ptr, uint64_t* nby
     return T2I_OK;
 }
 
+// The consumer's store (this) allocates pages for the producer's objects and
+// copies them page to page with the move kernel: source = the producer's
+// pages, destination = the new pages (§5.2: the consumer allocates a block in
+// its own arena and pulls the producer's bytes into it).
+t2i_status Store::pull_from(Store& src, const t2i_id* ids, uint32_t n, uint32_t consumers, t2i_id* out_ids,
+                            t2i_status* per_item, cudaStream_t stream) {
+    if (n == 0) return T2I_OK;
+    if (!ids || !out_ids) {
+        err_ = "pull: null id array";
+        return T2I_ERR_INVALID;
+    }
+    if (&src == this || src.device_ != device_ || src.page_shift_ != page_shift_) {
+        err_ = "pull: the stores must differ, share a device and have the same page size";
+        return T2I_ERR_INVALID;
+    }
+    // 1. every source id first (a failed pull changes nothing)
+    std::vector<const Object*> so(n);
+    t2i_status first = T2I_OK;
+    for (uint32_t i = 0; i < n; ++i) {
+        so[i] = src.ctl_.find(ids[i]);
+        t2i_status s = so[i] ? T2I_OK : (src.ctl_.is_evicted(ids[i]) ? T2I_ERR_EVICTED : T2I_ERR_NOT_FOUND);
+        if (s == T2I_ERR_EVICTED) src.ctl_.counters().misses++;
+        if (per_item) per_item[i] = s;
+        if (s != T2I_OK && first == T2I_OK) first = s;
+    }
+    if (first != T2I_OK) {
+        err_ = "pull: a source id is not in the producer's store";
+        return first;
+    }
+    // 2. room in this store, as intermediates
+    std::vector<t2i_put_desc> pd(n);
+    for (uint32_t i = 0; i < n; ++i)
+        pd[i] = t2i_put_desc{nullptr, so[i]->nbytes, 0, so[i]->dtype_tag, 0, 0, 0, consumers, 0};
+    t2i_status st = ctl_.put(pd.data(), n, out_ids, &objs_);
+    if (st != T2I_OK) {
+        err_ = ctl_.error();
+        return st;
+    }
+    // 3. the sources are read like a get
+    std::vector<t2i_get_desc> gd(n);
+    for (uint32_t i = 0; i < n; ++i) gd[i] = t2i_get_desc{ids[i], nullptr, 0, 0, 0};
+    std::vector<const Object*> src_objs;
+    src.ctl_.get(gd.data(), n, nullptr, &src_objs, /*defer_release=*/true);
+    // 4. page-to-page copies, after the producer's writer and this store's
+    //    earlier users of the new pages
+    DeviceGuard g(device_);
+    int sd = 0, ss = 0;
+    if ((st = stream_slot(stream, &sd)) != T2I_OK || (st = src.stream_slot(stream, &ss)) != T2I_OK) {
+        ctl_.rollback_put(out_ids, n);
+        src.ctl_.release_pending();
+        return st;
+    }
+    const uint64_t P = uint64_t(1) << page_shift_;
+    deps_.begin(sd);
+    src.deps_.begin(ss);
+    segs_.clear();
+    for (uint32_t i = 0; i < n; ++i) {
+        const Object* s_o = src_objs[i];
+        const Object* d_o = objs_[i];
+        for (size_t j = 0; j < s_o->pages.size(); ++j) {
+            src.deps_.reads(s_o->pages[j]);
+            deps_.writes(d_o->pages[j]);
+            segs_.push_back({src.pool_ + uint64_t(s_o->pages[j]) * P, std::min<uint64_t>(P, s_o->nbytes - j * P),
+                             &d_o->pages[j], 1u});
+        }
+    }
+    cudaError_t we = deps_.wait();
+    if (we == cudaSuccess) we = src.deps_.wait();
+    if (we != cudaSuccess) {
+        ctl_.rollback_put(out_ids, n);
+        src.ctl_.release_pending();
+        return cuda_fail("pull: cannot order after earlier calls", we);
+    }
+    if (!segs_.empty()) {
+        st = launch_segments<Mode::Move>(segs_, stream);
+        uint32_t qd = 0, qs = 0;
+        cudaError_t e1 = deps_.end(&qd);
+        cudaError_t e2 = src.deps_.end(&qs);
+        for (uint32_t i = 0; i < n; ++i) {
+            for (uint32_t pg : objs_[i]->pages) deps_.mark_write(pg, qd);
+            for (uint32_t pg : src_objs[i]->pages) src.deps_.mark_read(pg, qs);
+        }
+        if (st != T2I_OK) ctl_.rollback_put(out_ids, n);
+        else if (e1 != cudaSuccess || e2 != cudaSuccess)
+            st = cuda_fail("pull: cannot record its event", e1 != cudaSuccess ? e1 : e2);
+    }
+    src.ctl_.release_pending();
+    return st;
+}
+
 t2i_status Store::compact(uint64_t limit_bytes, cudaStream_t stream, uint64_t* moved) {
     std::vector<t2i_move> moves;
     t2i_status st = ctl_.compact(limit_bytes, &moves);
@@ -779,6 +871,22 @@ t2i_status t2i_put_layers(t2i_store* store, const t2i_put_desc* descs, const uin
 
 t2i_status t2i_view(t2i_store* store, t2i_id id, void* cuda_stream, void** dev_ptr, uint64_t* nbytes) {
     T2I_STORE_CALL(store, store->s->view(id, static_cast<cudaStream_t>(cuda_stream), dev_ptr, nbytes));
+}
+
+t2i_status t2i_pull(t2i_store* dst, t2i_store* src, const t2i_id* src_ids, uint32_t n, uint32_t consumers,
+                    t2i_id* out_ids, t2i_status* per_item, void* cuda_stream) {
+    if (!dst || !src) return T2I_ERR_INVALID;
+    if (dst == src) {
+        dst->s->set_error("pull: a store cannot pull from itself");
+        return T2I_ERR_INVALID;
+    }
+    std::scoped_lock lock(dst->s->mu, src->s->mu);
+    try {
+        return dst->s->pull_from(*src->s, src_ids, n, consumers, out_ids, per_item,
+                                 static_cast<cudaStream_t>(cuda_stream));
+    } catch (const std::bad_alloc&) {
+        return T2I_ERR_INVALID;
+    }
 }
 
 t2i_status t2i_compact(t2i_store* store, uint64_t limit_bytes, void* cuda_stream, uint64_t* pages_moved) {

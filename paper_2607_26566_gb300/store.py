@@ -250,6 +250,17 @@ class Store:
         ids = np.ascontiguousarray(ids, np.uint64)
         return self._lib.t2i_free(self._h, ids.ctypes.data_as(C.POINTER(C.c_uint64)), len(ids))
 
+    def pull(self, src: "Store", ids, consumers: int = 0, stream=None):
+        """(status, new ids, per-item statuses) -- t2i_pull: this store (the
+        consumer) pulls ``ids`` from the producer's store ``src``."""
+        ids = np.ascontiguousarray(ids, np.uint64)
+        out = np.zeros(len(ids), np.uint64)
+        per = np.zeros(len(ids), np.int32)
+        st = self._lib.t2i_pull(self._h, src._h, ids.ctypes.data_as(C.POINTER(C.c_uint64)), len(ids), consumers,
+                                out.ctypes.data_as(C.POINTER(C.c_uint64)), per.ctypes.data_as(C.POINTER(C.c_int32)),
+                                _stream(stream))
+        return st, out, per
+
     def view(self, oid: int, stream=None):
         """(status, device address, nbytes) -- t2i_view."""
         ptr = C.c_void_p()

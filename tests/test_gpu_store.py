@@ -543,3 +543,55 @@ def test_view_is_ordered_after_its_writer_and_before_reuse():
     assert s == 0 and st.ctl.object(int(iy))[2] == list(range(8))
     torch.cuda.synchronize()
     assert torch.equal(z, x)
+
+
+def test_pull_between_stores_vs_oracle():
+    """A consumer's store pulls objects from a producer's store page to page
+    (§5.2): statuses, ids, placement and bytes as the oracle's pull."""
+    P = 64 * 1024
+    rng = np.random.default_rng(21)
+    prod, cons = make_store(64 * P, P), make_store(16 * P, P, alloc_policy=1)
+    o_prod, o_cons = OracleStore(64 * P, P), OracleStore(16 * P, P, policy=1)
+    datas = [rng.integers(0, 256, int(n), dtype=np.uint8) for n in (3 * P + 11, 1000, 5 * P, 17, 2 * P)]
+    cons_n = [1, 0, 0, 2, 0]
+    s, ids = prod.put_batch(put_descs([dev_bytes(d) for d in datas], dtype_tag=2, consumers=cons_n))
+    assert s == 0
+    _, oids = o_prod.put_batch([PutItem(d.size, d, 2, 0, 0, False, c) for d, c in zip(datas, cons_n)])
+    pick = [int(ids[0]), int(ids[2]), int(ids[3])]
+    s, new, per = cons.pull(prod, pick, consumers=1)
+    ost, oper, onew = o_cons.pull(o_prod, pick, consumers=1)
+    assert s == ost == 0 and list(per) == oper and list(new) == onew
+    compare_meta(cons, o_cons)
+    compare_meta(prod, o_prod)
+    assert prod.stats()["reclaimed"] == o_prod.stats["reclaimed"] == 1   # object 0's only consumer was the pull
+    outs = [dev_empty(datas[i].size) for i in (0, 2, 3)]
+    assert cons.get_batch(get_descs([int(x) for x in new], outs))[0] == 0
+    torch.cuda.synchronize()
+    for o, i in zip(outs, (0, 2, 3)):
+        assert np.array_equal(host(o), datas[i])
+    assert cons.stats()["reclaimed"] == 3                                # consumers = 1 each
+    # failures change nothing
+    assert cons.pull(prod, [int(ids[0])])[0] == 3                       # reclaimed in the producer
+    big = dev_bytes(rng.integers(0, 256, 17 * P, dtype=np.uint8))
+    s, (ib,) = prod.put_batch(put_descs([big]))
+    assert cons.pull(prod, [int(ib)])[0] == 2 and prod.ctl.object(int(ib))[0] == 0
+    assert cons.pull(cons, [int(ib)])[0] == 1
+    other = make_store(16 * 4096, 4096)
+    assert other.pull(prod, [int(ib)])[0] == 1                          # page sizes differ
+
+
+def test_pull_waits_for_a_late_producer():
+    P = 64 * 1024
+    prod, cons = make_store(16 * P, P), make_store(16 * P, P)
+    s1, s2 = torch.cuda.Stream(), torch.cuda.Stream()
+    x = torch.randint(0, 256, (9 * P + 3,), dtype=torch.uint8, device=DEV)
+    torch.cuda.synchronize()
+    _late(s1, 30)
+    s, (ix,) = prod.put_batch(put_descs([x]), stream=s1)
+    assert s == 0
+    s, (iy,), _ = cons.pull(prod, [int(ix)], stream=s2)
+    assert s == 0
+    out = torch.zeros_like(x)
+    assert cons.get_batch(get_descs([int(iy)], [out]), stream=s2)[0] == 0
+    torch.cuda.synchronize()
+    assert torch.equal(out, x)

@@ -452,3 +452,26 @@ def test_planted_best_fit_is_caught(monkeypatch):
         return run
     monkeypatch.setattr(OracleStore, "_take_pages", take)
     assert _expect_failure(test_extent_policy_hand_trace)
+
+
+def test_pull_hand_trace():
+    """Reading 11 (§5.2): the consumer's store allocates and copies; the
+    producer's object is read like a get."""
+    P = 256
+    prod = OracleStore(8 * P, P, paged_pool=True)
+    cons = OracleStore(4 * P, P, paged_pool=True)
+    a = np.arange(600, dtype=np.uint8)
+    _, (ia,) = prod.put_batch([PutItem(600, a, dtype_tag=3, group=7, consumers=1)])
+    st, per, (ic,) = cons.pull(prod, [ia], consumers=2)
+    assert st == OK and per == [OK] and cons.pages_of(ic) == [0, 1, 2]
+    o = cons.objects[ic]
+    assert (o.dtype_tag, o.group, o.evictable, o.consumers_left) == (3, 0, False, 2)
+    assert ia not in prod.objects and prod.stats["reclaimed"] == 1   # its one consumer was the pull
+    _, _, (out,) = cons.get_batch([ic])
+    assert np.array_equal(out, a)
+    st, per, _ = cons.pull(prod, [ia])
+    assert st == NOT_FOUND and per == [NOT_FOUND]
+    _, (ib,) = prod.put_batch([PutItem(600, a)])
+    assert cons.pull(prod, [ib])[0] == NOSPACE and ib in prod.objects  # 3 + 3 pages > 4: nothing happens
+    assert prod.objects[ib].consumers_left == 0
+    assert cons.pull(OracleStore(4 * 128, 128), [1])[0] == INVALID        # page sizes differ
