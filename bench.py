@@ -957,13 +957,21 @@ def time_pull(device, B: int = 8, requests: int = 64, reps: int = 3):
         hw.ids[n * r:n * (r + 1)] = ids
     payload = sum(sp.nbytes for sp in hw.specs) * requests
 
+    # raw C-ABI calls with arrays built once (the binding's per-call array
+    # allocations would make the host, not the GPU, the bottleneck)
+    lib = cons._lib
+    new = np.zeros(requests * n, np.uint64)
+    src_p = [C.cast(C.c_void_p(hw.ids.ctypes.data + 8 * n * r), C.POINTER(C.c_uint64)) for r in range(requests)]
+    dst_p = [C.cast(C.c_void_p(new.ctypes.data + 8 * n * r), C.POINTER(C.c_uint64)) for r in range(requests)]
+    new_all = new.ctypes.data_as(C.POINTER(C.c_uint64))
+    s_h = C.c_void_p(stream.cuda_stream)
+
     def once():
-        new = []
         for r in range(requests):
-            st, out, _ = cons.pull(hw.store, hw.ids[n * r:n * (r + 1)])
-            cons.check(st)
-            new.append(out)
-        cons.check(cons.free(np.concatenate(new)))
+            st = lib.t2i_pull(cons._h, hw.store._h, src_p[r], n, 0, dst_p[r], None, s_h)
+            if st:
+                raise RuntimeError("pull: " + cons.last_error())
+        cons.check(lib.t2i_free(cons._h, new_all, len(new)))
 
     once()
     torch.cuda.synchronize(device)
