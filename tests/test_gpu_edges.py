@@ -1,0 +1,115 @@
+"""Edge cases of the launch packing on the GPU (marked gpu): an object whose
+page list is longer than one launch's parameter space, a batch whose
+descriptors span several launches, 1 GiB pages, empty and zero-byte batches,
+and both unaligned kernels; all compared with the oracle's get."""
+import numpy as np
+import pytest
+import torch
+
+from oracle import OracleStore, PutItem
+from oracle.cast import f32_bits_to_bf16_bits
+from paper_2607_26566_gb300 import Store, get_descs, put_descs
+
+pytestmark = pytest.mark.gpu
+DEV = torch.device("cuda", 0)
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _built(lib):
+    assert torch.cuda.is_available(), "GPU tests need a CUDA device"
+    yield
+
+
+def store(pool_bytes, page_bytes, **kw):
+    return Store(torch.empty(pool_bytes, dtype=torch.uint8, device=DEV), page_bytes, **kw)
+
+
+def test_object_longer_than_one_launch():
+    """8,000 pages of 256 B: the page list is split across launches."""
+    P = 256
+    st = store(9000 * P, P)
+    x = torch.randint(0, 256, (8000 * P - 77,), dtype=torch.uint8, device=DEV)
+    s, (i,) = st.put_batch(put_descs([x]))
+    assert s == 0 and st.stats()["launches"] >= 2
+    out = torch.zeros_like(x)
+    l0 = st.stats()["launches"]
+    assert st.get_batch(get_descs([int(i)], [out]))[0] == 0
+    assert st.stats()["launches"] - l0 >= 2
+    torch.cuda.synchronize()
+    assert torch.equal(out, x)
+
+
+def test_batch_spanning_several_launches():
+    """1,500 objects in one call: descriptors for several launches; every
+    object's bytes and every page list as the oracle's."""
+    P = 4096
+    rng = np.random.default_rng(8)
+    st = store(4000 * P, P)
+    ora = OracleStore(4000 * P, P)
+    sizes = rng.integers(1, 2 * P + 1, 1500)
+    buf = torch.randint(0, 256, (int(sizes.sum()) + 16,), dtype=torch.uint8, device=DEV)
+    offs = np.concatenate([[0], np.cumsum(sizes)[:-1]])
+    s, ids = st.put_batch(put_descs(buf.data_ptr() + offs, nbytes=sizes))
+    assert s == 0 and st.stats()["launches"] >= 2
+    host = buf.cpu().numpy()
+    _, oids = ora.put_batch([PutItem(int(n), host[o:o + n]) for o, n in zip(offs, sizes)])
+    assert list(ids) == oids
+    out = torch.zeros(int(sizes.sum()) + 64 * 1500, dtype=torch.uint8, device=DEV)
+    doffs = np.concatenate([[0], np.cumsum(sizes + 64)[:-1]]) + 3     # unaligned destinations
+    assert st.get_batch(get_descs(ids, out.data_ptr() + doffs, dst_bytes=sizes))[0] == 0
+    torch.cuda.synchronize()
+    got = out.cpu().numpy()
+    _, _, want = ora.get_batch(oids)
+    for d, n, w in zip(doffs, sizes, want):
+        assert np.array_equal(got[d:d + n], w)
+    for oid in oids[::97]:
+        assert st.ctl.object(oid)[2] == ora.objects[oid].pages
+
+
+def test_gigabyte_pages():
+    P = 1 << 30
+    st = store(2 * P, P)
+    x = torch.randint(0, 256, (P + P // 2 + 5,), dtype=torch.uint8, device=DEV)
+    s, (i,) = st.put_batch(put_descs([x]))
+    assert s == 0 and st.ctl.object(int(i))[2] == [0, 1]
+    out = torch.empty_like(x)
+    assert st.get_batch(get_descs([int(i)], [out]))[0] == 0
+    torch.cuda.synchronize()
+    assert torch.equal(out, x)
+    del x, out
+
+
+def test_empty_and_zero_byte_batches():
+    P = 4096
+    st = store(16 * P, P)
+    assert st.put_batch(put_descs([]))[0] == 0
+    assert st.get_batch(get_descs([]))[0] == 0
+    assert st.free([]) == 0
+    s, ids = st.put_batch(put_descs([0, 0, 0], nbytes=[0, 0, 0]))
+    assert s == 0 and len(ids) == 3 and st.stats()["launches"] == 0
+    assert st.get_batch(get_descs(ids, [0, 0, 0], dst_bytes=[0, 0, 0]))[0] == 0
+    assert st.stats()["launches"] == 0 and st.stats()["used_pages"] == 0
+
+
+def test_unaligned_cast_and_copy_kernels():
+    """Sources at every 16-byte misalignment (put), destinations at every
+    misalignment (copy) and every even one (cast): the any-alignment kernels."""
+    P = 8192
+    st = store(512 * P, P)
+    rng = np.random.default_rng(2)
+    f = rng.standard_normal(3 * P // 4 + 13).astype(np.float32)
+    for m in range(16):
+        raw = torch.zeros(f.nbytes + 32, dtype=torch.uint8, device=DEV)
+        raw[m:m + f.nbytes].copy_(torch.from_numpy(f.view(np.uint8)))
+        s, (i,) = st.put_batch(put_descs([raw.data_ptr() + m], nbytes=[f.nbytes]))
+        assert s == 0
+        out = torch.zeros(f.nbytes + 32, dtype=torch.uint8, device=DEV)
+        assert st.get_batch(get_descs([int(i)], [out.data_ptr() + (15 - m)], dst_bytes=[f.nbytes]))[0] == 0
+        bf = torch.zeros(f.nbytes // 2 + 32, dtype=torch.uint8, device=DEV)
+        e = 2 * (m % 8)
+        assert st.get_batch(get_descs([int(i)], [bf.data_ptr() + e], dst_bytes=[f.nbytes // 2], cast=1))[0] == 0
+        torch.cuda.synchronize()
+        assert np.array_equal(out.cpu().numpy()[15 - m:15 - m + f.nbytes], f.view(np.uint8))
+        got = bf.cpu().numpy()[e:e + f.nbytes // 2].view(np.uint16)
+        assert np.array_equal(got, f32_bits_to_bf16_bits(f.view(np.uint32)))
+        assert st.free([int(i)]) == 0
