@@ -163,8 +163,8 @@ t2i_status t2i_store_destroy(t2i_store* store);
  * Returns NOSPACE (and evicts nothing) if even that is not enough, INVALID
  * for a bad descriptor; out_ids[i] receives the id of descs[i] (n ids).
  * The copy is one kernel launch per batch (more only when the descriptors
- * exceed one launch's parameter space). On CUDA the batch is not stored;
- * evictions it made stand.                                                   */
+ * exceed one launch's parameter space). On CUDA the batch is not stored
+ * (pages, ids and counters as before the call); evictions it made stand.     */
 t2i_status t2i_put_batch(t2i_store* store, const t2i_put_desc* descs, uint32_t n, t2i_id* out_ids,
                          void* cuda_stream);
 
@@ -275,6 +275,13 @@ t2i_status t2i_ctl_free_pages(const t2i_ctl* ctl, uint32_t* out, uint64_t cap, u
 t2i_status t2i_ctl_last_evictions(const t2i_ctl* ctl, t2i_id* out, uint64_t cap, uint64_t* n);
 t2i_status t2i_ctl_stats(const t2i_ctl* ctl, t2i_stats* out);
 const char* t2i_ctl_last_error(const t2i_ctl* ctl);
+
+/* Testing support: the countdown-th kernel launch of this store from now
+ * reports T2I_ERR_CUDA without being issued (0 cancels). It exercises the
+ * store's recovery on the host -- a put is rolled back (pages, ids and
+ * counters as before it; evictions stand), a get counts nothing, a compaction
+ * restores its page tables and limit -- without faulting a GPU.            */
+t2i_status t2i_inject_launch_failure(t2i_store* store, uint32_t countdown);
 
 /* =========================================================================
  * First-layer prefix caching (§5.1). A model of L layers keeps its first L_e

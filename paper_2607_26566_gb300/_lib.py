@@ -69,6 +69,7 @@ PROTOTYPES = {
     "t2i_pull": (_S, [_P, _P, _PU64, _U32, _U32, _PU64, C.POINTER(_S), _P]),
     "t2i_free": (_S, [_P, _PU64, _U32]),
     "t2i_compact": (_S, [_P, _U64, _P, _PU64]),
+    "t2i_inject_launch_failure": (_S, [_P, _U32]),
     "t2i_store_stats": (_S, [_P, C.POINTER(Stats)]),
     "t2i_store_ctl": (_P, [_P]),
     "t2i_last_error": (C.c_char_p, [_P]),

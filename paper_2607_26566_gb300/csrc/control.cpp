@@ -100,10 +100,13 @@ void FreePages::insert_page(uint32_t p) {
     }
 }
 
-void FreePages::give(const std::vector<uint32_t>& pages) {
+void FreePages::give(const std::vector<uint32_t>& pages, bool undo) {
     count_ += pages.size();
     if (policy_ == 0) {
-        for (uint32_t p : pages) stack_.push_back(p);
+        if (undo)
+            for (size_t j = pages.size(); j-- > 0;) stack_.push_back(pages[j]);
+        else
+            for (uint32_t p : pages) stack_.push_back(p);
         return;
     }
     for (uint32_t p : pages) insert_page(p);
@@ -242,6 +245,16 @@ t2i_status Control::view(uint64_t id, const Object** out) {
     return T2I_OK;
 }
 
+void Control::rollback_compact() {
+    for (const Remap& r : last_remap_) r.o->pages[r.idx] = r.old_page;
+    last_remap_.clear();
+    free_.restore(std::move(last_free_));
+    last_free_ = FreePages::Snapshot{};
+    limit_pages_ = last_limit_;
+    counters_.pages_moved = last_compact_counters_.pages_moved;
+    counters_.bytes_moved = last_compact_counters_.bytes_moved;
+}
+
 const Object* Control::find(uint64_t id) const {
     const uintptr_t v = ids_.get(id);
     return v > IdTable::kEvicted ? reinterpret_cast<const Object*>(v) : nullptr;
@@ -339,13 +352,49 @@ t2i_status Control::put(const t2i_put_desc* descs, uint32_t n, t2i_id* ids, std:
 }
 
 void Control::rollback_put(const t2i_id* ids, uint32_t n) {
-    for (uint32_t i = 0; i < n; ++i) {
+    // last object first, each object's pages in reverse: the exact undo of
+    // the pops that placed them
+    for (uint32_t i = n; i-- > 0;) {
         Object* o = const_cast<Object*>(find(ids[i]));
         if (!o) continue;
         counters_.puts--;
         counters_.bytes_put -= o->nbytes;
-        release(o, false);
+        const uint64_t np = o->pages.size();
+        free_.give(o->pages, /*undo=*/true);
+        used_pages_ -= np;
+        Group* g = o->group;
+        g->n_objects--;
+        if (o->evictable) {
+            g->victims.erase({o->order, o->id});
+            g->evictable_pages -= np;
+            evictable_pages_ -= np;
+            if (g->victims.empty() && g->rec_key) {
+                recency_.erase({g->rec_key, g});
+                g->rec_key = 0;
+            }
+        }
+        const size_t li = o->live_index;
+        live_[li] = live_.back();
+        live_[li]->live_index = li;
+        live_.pop_back();
+        ids_.clear(o->id, next_id_);
+        if (o->id + 1 == next_id_) next_id_ = o->id;  // never handed out: issue again
+        delete o;
+        maybe_drop_group(g);
     }
+}
+
+void Control::account_get(const t2i_id* ids, uint32_t n, size_t stride) {
+    const char* base = reinterpret_cast<const char*>(ids);
+    for (uint32_t i = 0; i < n; ++i) {
+        const t2i_id id = *reinterpret_cast<const t2i_id*>(base + i * stride);
+        Object* o = reinterpret_cast<Object*>(ids_.get(id));
+        touch(o);
+        counters_.gets++;
+        counters_.bytes_got += o->nbytes;
+        if (o->consumers_left > 0 && --o->consumers_left == 0) pending_release_.push_back(o);
+    }
+    flush_touches();
 }
 
 t2i_status Control::get(const t2i_get_desc* descs, uint32_t n, t2i_status* per_item,
@@ -388,14 +437,10 @@ t2i_status Control::get(const t2i_get_desc* descs, uint32_t n, t2i_status* per_i
         err_ = "get: item " + std::to_string(first_i) + ": " + what[first];
         return first;
     }
-    for (uint32_t i = 0; i < n; ++i) {
-        Object* o = reinterpret_cast<Object*>(ids_.get(descs[i].id));
-        touch(o);
-        counters_.gets++;
-        counters_.bytes_got += o->nbytes;
-        if (o->consumers_left > 0 && --o->consumers_left == 0) pending_release_.push_back(o);
+    if (objs) {
+        for (uint32_t i = 0; i < n; ++i) (*objs)[i] = reinterpret_cast<const Object*>(ids_.get(descs[i].id));
     }
-    flush_touches();
+    account_get(&descs[0].id, n, sizeof(t2i_get_desc));
     if (!defer_release) release_pending();
     return T2I_OK;
 }
@@ -465,6 +510,11 @@ t2i_status Control::compact(uint64_t limit_bytes, std::vector<t2i_move>* moves) 
     }
     std::sort(tail.begin(), tail.end(), [](const Tail& a, const Tail& b) { return a.page < b.page; });
     moves->reserve(tail.size());
+    last_remap_.clear();
+    last_remap_.reserve(tail.size());
+    last_free_ = free_.snapshot();
+    last_limit_ = limit_pages_;
+    last_compact_counters_ = counters_;
     uint64_t scan = 0;
     uint64_t moved_bytes = 0;
     for (const Tail& t : tail) {
@@ -473,6 +523,7 @@ t2i_status Control::compact(uint64_t limit_bytes, std::vector<t2i_move>* moves) 
         used[scan] = 1;
         const uint64_t valid = std::min<uint64_t>(P_, t.o->nbytes - uint64_t(t.idx) * P_);
         t.o->pages[t.idx] = dst;
+        last_remap_.push_back({t.o, t.idx, t.page});
         moves->push_back({t.page, dst, valid});
         moved_bytes += valid;
     }

@@ -76,8 +76,21 @@ class FreePages {
     uint32_t policy() const { return policy_; }
     // k pages for one object, in page-list order (requires k <= size())
     void take(uint64_t k, std::vector<uint32_t>* out);
-    // an object's pages back, in page-list order
-    void give(const std::vector<uint32_t>& pages);
+    // an object's pages back, in page-list order (or, undoing a take, in
+    // reverse, which restores a LIFO stack exactly)
+    void give(const std::vector<uint32_t>& pages, bool undo = false);
+    // the whole structure, for undoing a compaction
+    struct Snapshot {
+        uint64_t count;
+        std::vector<uint32_t> stack;
+        std::map<uint32_t, uint32_t> runs;
+    };
+    Snapshot snapshot() const { return {count_, stack_, runs_}; }
+    void restore(Snapshot s) {
+        count_ = s.count;
+        stack_ = std::move(s.stack);
+        runs_ = std::move(s.runs);
+    }
     // after a compaction: every page below limit that `used` does not mark
     void rebuild(uint64_t limit, const std::vector<uint8_t>& used);
     // policy 0: the stack from bottom to top; policy 1: ascending
@@ -127,8 +140,14 @@ class Control {
     // put: validates, evicts, allocates and commits. On success ids[i] and
     // created[i] (if non-null) describe descs[i].
     t2i_status put(const t2i_put_desc* descs, uint32_t n, t2i_id* ids, std::vector<const Object*>* created);
-    // Undo the put of freshly created objects (after a failed launch).
+    // Undo the put of freshly created objects (after a failed launch):
+    // pages, ids and counters return to their state before the put;
+    // evictions it made and recency stamps stand.
     void rollback_put(const t2i_id* ids, uint32_t n);
+    // The accounting half of a get (recency stamps, consumer counts) for
+    // items already validated; objects consumed to zero wait for
+    // release_pending(). Called after the get's copies are enqueued.
+    void account_get(const t2i_id* ids, uint32_t n, size_t stride);
     // get: validates every item (per_item nullable), then stamps recency and
     // counts consumers. objs[i] receives the object of descs[i] on success.
     // dst fields are not looked at here. Objects whose last consumer this was
@@ -140,6 +159,9 @@ class Control {
     t2i_status free(const t2i_id* ids, uint32_t n);
     // compact: plans, remaps and returns the moves (always filled).
     t2i_status compact(uint64_t limit_bytes, std::vector<t2i_move>* moves);
+    // Undo the last compaction (after a failed launch): page lists, the free
+    // pages and the limit return to their state before it.
+    void rollback_compact();
 
     uint64_t live_pages_at_or_above(uint64_t limit) const;
     const Object* find(uint64_t id) const;
@@ -179,6 +201,15 @@ class Control {
     std::vector<Group*> touched_;
     std::vector<t2i_id> last_evictions_;
     std::vector<Object*> pending_release_;   // consumed to zero by the last get
+    struct Remap {
+        Object* o;
+        uint32_t idx;
+        uint32_t old_page;
+    };
+    std::vector<Remap> last_remap_;          // the last compaction, for rollback_compact
+    FreePages::Snapshot last_free_;
+    uint64_t last_limit_ = 0;
+    t2i_stats last_compact_counters_{};
     t2i_stats counters_{};
     std::string err_;
 };

@@ -143,6 +143,7 @@ class Store {
     Control& ctl() { return ctl_; }
     const std::string& error() const { return err_; }
     void set_error(std::string e) { err_ = std::move(e); }
+    void inject_launch_failure(uint32_t countdown) { fail_countdown_ = countdown; }
 
     t2i_status put(const t2i_put_desc* descs, uint32_t n, t2i_id* ids, cudaStream_t stream);
     t2i_status get(const t2i_get_desc* descs, uint32_t n, t2i_status* per_item, cudaStream_t stream,
@@ -201,6 +202,7 @@ class Store {
     t2i_ctl handle_{};
     uint32_t page_shift_ = 0;
     int max_ctas_[3][2] = {{1, 1}, {1, 1}, {1, 1}};  // [mode][any alignment]: resident CTAs on the device
+    uint32_t fail_countdown_ = 0;  // > 0: that many launches from now, report a failure (testing)
     std::vector<Seg> aligned_, general_;
     StreamDeps deps_;
     std::string err_;
@@ -300,6 +302,10 @@ t2i_status Store::launch_one(const std::vector<SegDesc>& sd, const std::vector<u
     const void* fn = M == Mode::Put   ? reinterpret_cast<const void*>(scatter_put_kernel<BLOB, GENERAL>)
                      : M == Mode::Get ? reinterpret_cast<const void*>(gather_get_kernel<BLOB, GENERAL>)
                                       : reinterpret_cast<const void*>(compact_move_kernel<BLOB>);
+    if (fail_countdown_ && --fail_countdown_ == 0) {
+        err_ = "kernel launch failed: injected failure (t2i_inject_launch_failure)";
+        return T2I_ERR_CUDA;
+    }
     cudaLaunchConfig_t lc = {};
     lc.gridDim = dim3(grid);
     lc.blockDim = dim3(kThreads);
@@ -530,27 +536,17 @@ t2i_status Store::get(const t2i_get_desc* descs, uint32_t n, t2i_status* per_ite
                (first == T2I_ERR_INVALID && !why.empty() ? " (" + why + ")" : "");
         return first;
     }
-    // 2. LRU stamps and consumer counts (objects consumed to zero are freed
-    //    after their pages have been packed into this call's launches)
-    t2i_status st = ctl_.get(descs, n, per_item, &objs_, /*defer_release=*/true);
-    if (st != T2I_OK) {
-        err_ = ctl_.error();
-        return st;
-    }
-    // 3. one gather launch for the batch (copies and casts together), after
+    // 2. one gather launch for the batch (copies and casts together), after
     //    the calls that wrote its pages and after the caller's event
+    objs_.resize(n);
+    for (uint32_t i = 0; i < n; ++i) objs_[i] = ctl_.find(descs[i].id);
     DeviceGuard g(device_);
     int si = 0;
-    if ((st = stream_slot(stream, &si)) != T2I_OK) {
-        ctl_.release_pending();
-        return st;
-    }
+    t2i_status st = stream_slot(stream, &si);
+    if (st != T2I_OK) return st;
     if (wait_event) {
         cudaError_t e = cudaStreamWaitEvent(stream, wait_event, 0);
-        if (e != cudaSuccess) {
-            ctl_.release_pending();
-            return cuda_fail("get: cannot wait for the event", e);
-        }
+        if (e != cudaSuccess) return cuda_fail("get: cannot wait for the event", e);
     }
     segs_.clear();
     deps_.begin(si);
@@ -563,18 +559,21 @@ t2i_status Store::get(const t2i_get_desc* descs, uint32_t n, t2i_status* per_ite
     }
     if (!segs_.empty()) {
         cudaError_t we = deps_.wait();
-        if (we != cudaSuccess) {
-            ctl_.release_pending();
-            return cuda_fail("get: cannot order after earlier calls", we);
-        }
+        if (we != cudaSuccess) return cuda_fail("get: cannot order after earlier calls", we);
         st = launch_segments<Mode::Get>(segs_, stream);
+        if (st != T2I_OK) return st;  // nothing was counted: the get did not happen
         uint32_t q = 0;
         cudaError_t ee = deps_.end(&q);
         for (const Seg& sg : segs_)
             for (uint32_t k = 0; k < sg.n_pages; ++k) deps_.mark_read(sg.pages[k], q);
-        if (st == T2I_OK && ee != cudaSuccess) st = cuda_fail("get: cannot record its event", ee);
+        if (ee != cudaSuccess) st = cuda_fail("get: cannot record its event", ee);
     }
-    ctl_.release_pending();  // objects consumed to zero: their pages carry this call as a reader
+    // 3. LRU stamps and consumer counts, now that the copies are enqueued;
+    //    objects consumed to zero are freed (their pages carry this call as
+    //    a reader, so reuse waits for it)
+    if (per_item) std::fill(per_item, per_item + n, T2I_OK);
+    ctl_.account_get(&descs[0].id, n, sizeof(t2i_get_desc));
+    ctl_.release_pending();
     return st;
 }
 
@@ -643,18 +642,13 @@ t2i_status Store::pull_from(Store& src, const t2i_id* ids, uint32_t n, uint32_t 
         err_ = ctl_.error();
         return st;
     }
-    // 3. the sources are read like a get
-    std::vector<t2i_get_desc> gd(n);
-    for (uint32_t i = 0; i < n; ++i) gd[i] = t2i_get_desc{ids[i], nullptr, 0, 0, 0};
-    std::vector<const Object*> src_objs;
-    src.ctl_.get(gd.data(), n, nullptr, &src_objs, /*defer_release=*/true);
-    // 4. page-to-page copies, after the producer's writer and this store's
+    const std::vector<const Object*>& src_objs = so;
+    // 3. page-to-page copies, after the producer's writer and this store's
     //    earlier users of the new pages
     DeviceGuard g(device_);
     int sd = 0, ss = 0;
     if ((st = stream_slot(stream, &sd)) != T2I_OK || (st = src.stream_slot(stream, &ss)) != T2I_OK) {
         ctl_.rollback_put(out_ids, n);
-        src.ctl_.release_pending();
         return st;
     }
     const uint64_t P = uint64_t(1) << page_shift_;
@@ -675,11 +669,14 @@ t2i_status Store::pull_from(Store& src, const t2i_id* ids, uint32_t n, uint32_t 
     if (we == cudaSuccess) we = src.deps_.wait();
     if (we != cudaSuccess) {
         ctl_.rollback_put(out_ids, n);
-        src.ctl_.release_pending();
         return cuda_fail("pull: cannot order after earlier calls", we);
     }
     if (!segs_.empty()) {
         st = launch_segments<Mode::Move>(segs_, stream);
+        if (st != T2I_OK) {
+            ctl_.rollback_put(out_ids, n);  // the sources were not read: nothing counted
+            return st;
+        }
         uint32_t qd = 0, qs = 0;
         cudaError_t e1 = deps_.end(&qd);
         cudaError_t e2 = src.deps_.end(&qs);
@@ -687,10 +684,11 @@ t2i_status Store::pull_from(Store& src, const t2i_id* ids, uint32_t n, uint32_t 
             for (uint32_t pg : objs_[i]->pages) deps_.mark_write(pg, qd);
             for (uint32_t pg : src_objs[i]->pages) src.deps_.mark_read(pg, qs);
         }
-        if (st != T2I_OK) ctl_.rollback_put(out_ids, n);
-        else if (e1 != cudaSuccess || e2 != cudaSuccess)
+        if (e1 != cudaSuccess || e2 != cudaSuccess)
             st = cuda_fail("pull: cannot record its event", e1 != cudaSuccess ? e1 : e2);
     }
+    // 4. the sources are read like a get (stamps, consumer counts)
+    src.ctl_.account_get(ids, n, sizeof(t2i_id));
     src.ctl_.release_pending();
     return st;
 }
@@ -713,13 +711,23 @@ t2i_status Store::compact(uint64_t limit_bytes, cudaStream_t stream, uint64_t* m
         deps_.writes(m.dst_page);
     }
     cudaError_t we = deps_.wait();
-    if (we != cudaSuccess) return cuda_fail("compact: cannot order after earlier calls", we);
+    if (we != cudaSuccess) {
+        ctl_.rollback_compact();
+        if (moved) *moved = 0;
+        return cuda_fail("compact: cannot order after earlier calls", we);
+    }
     segs_.clear();
     const uint64_t P = uint64_t(1) << page_shift_;
     // each move is a one-page segment whose source is the old page
     for (const t2i_move& m : moves)
         segs_.push_back({pool_ + uint64_t(m.src_page) * P, m.valid_bytes, &m.dst_page, 1u});
     st = launch_segments<Mode::Move>(segs_, stream);
+    if (st != T2I_OK) {
+        // the old pages still hold every byte: point the page tables back
+        ctl_.rollback_compact();
+        if (moved) *moved = 0;
+        return st;
+    }
     uint32_t q = 0;
     cudaError_t ee = deps_.end(&q);
     for (const t2i_move& m : moves) {
@@ -891,6 +899,13 @@ t2i_status t2i_pull(t2i_store* dst, t2i_store* src, const t2i_id* src_ids, uint3
 
 t2i_status t2i_compact(t2i_store* store, uint64_t limit_bytes, void* cuda_stream, uint64_t* pages_moved) {
     T2I_STORE_CALL(store, store->s->compact(limit_bytes, static_cast<cudaStream_t>(cuda_stream), pages_moved));
+}
+
+t2i_status t2i_inject_launch_failure(t2i_store* store, uint32_t countdown) {
+    if (!store) return T2I_ERR_INVALID;
+    std::lock_guard<std::mutex> lock(store->s->mu);
+    store->s->inject_launch_failure(countdown);
+    return T2I_OK;
 }
 
 t2i_status t2i_store_stats(const t2i_store* store, t2i_stats* out) {

@@ -308,6 +308,10 @@ class Store:
         st = self._lib.t2i_compact(self._h, limit_bytes, _stream(stream), C.byref(n))
         return st, int(n.value)
 
+    def inject_launch_failure(self, countdown: int) -> int:
+        """t2i_inject_launch_failure (testing)."""
+        return self._lib.t2i_inject_launch_failure(self._h, countdown)
+
     def stats(self) -> dict:
         s = L.Stats()
         st = self._lib.t2i_store_stats(self._h, C.byref(s))
