@@ -95,7 +95,7 @@ def build(verbose: bool = False, ptxas_info: bool = False, defines=(), out: str 
     if errors:
         raise RuntimeError("compilation failed:\n" + "\n".join(errors))
     tmp = lib_path + ".tmp"
-    link = [nvcc, "-shared", *ARCH, "-o", tmp, *objs, "-cudart", "static", "-lpthread",
+    link = [nvcc, "-shared", *ARCH, "-o", tmp, *objs, "-cudart", "static", "-lpthread", "-ldl",
             "-Xlinker", "--version-script=" + os.path.join(CSRC, "exports.map")]
     r = subprocess.run(link, stdout=subprocess.PIPE, stderr=subprocess.STDOUT, text=True)
     if verbose or r.returncode:

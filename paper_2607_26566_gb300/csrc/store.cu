@@ -2,6 +2,7 @@
 // t2i_store / t2i_put_batch / t2i_get_batch / t2i_free / t2i_compact C ABI.
 #include <cuda.h>
 #include <cuda_runtime.h>
+#include <nvtx3/nvToolsExt.h>
 
 #include <algorithm>
 #include <cstring>
@@ -87,6 +88,13 @@ struct DeviceGuard {
     ~DeviceGuard() {
         if (switched) cudaSetDevice(prev);
     }
+};
+
+// One NVTX range per library call, named after it (profilers show the host
+// control around the launches; without a tool attached it costs a branch).
+struct NvtxRange {
+    explicit NvtxRange(const char* name) { nvtxRangePushA(name); }
+    ~NvtxRange() { nvtxRangePop(); }
 };
 
 int log2_exact(uint64_t v) {
@@ -813,6 +821,7 @@ t2i_status t2i_store_destroy(t2i_store* store) {
 #define T2I_STORE_CALL(store, expr)                                   \
     do {                                                              \
         if (!(store)) return T2I_ERR_INVALID;                         \
+        t2i::NvtxRange nvtx_range(__func__);                          \
         std::lock_guard<std::mutex> lock((store)->s->mu);             \
         try {                                                         \
             return (expr);                                            \
@@ -853,6 +862,7 @@ t2i_status t2i_put_layers(t2i_store* store, const t2i_put_desc* descs, const uin
             return T2I_ERR_INVALID;
         }
     }
+    t2i::NvtxRange nvtx_range("t2i_put_layers");
     cudaStream_t stream = static_cast<cudaStream_t>(cuda_stream);
     for (uint32_t l = first; l < n_layers; ++l) {
         t2i_status st;
@@ -888,6 +898,7 @@ t2i_status t2i_pull(t2i_store* dst, t2i_store* src, const t2i_id* src_ids, uint3
         dst->s->set_error("pull: a store cannot pull from itself");
         return T2I_ERR_INVALID;
     }
+    t2i::NvtxRange nvtx_range("t2i_pull");
     std::scoped_lock lock(dst->s->mu, src->s->mu);
     try {
         return dst->s->pull_from(*src->s, src_ids, n, consumers, out_ids, per_item,
