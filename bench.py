@@ -470,9 +470,24 @@ def time_weights(device, reps: int = 3, h2d_mode: int = 0):
     launches = (wr.store.stats()["launches"] - launches0) / reps
     ok = wr.verify()
     pm, gm, gk = statistics.median(put_ms), statistics.median(get_ms), statistics.median(get_kern_ms)
+    # the host link's ceiling on this machine: a plain pinned copy (torch) of 1 GiB
+    hb = torch.empty(1 << 30, dtype=torch.uint8).pin_memory()
+    db = torch.empty(1 << 30, dtype=torch.uint8, device=device)
+    db.copy_(hb, non_blocking=True)
+    torch.cuda.synchronize(device)
+    e[0].record(stream)
+    for _ in range(3):
+        db.copy_(hb, non_blocking=True)
+    e[1].record(stream)
+    torch.cuda.synchronize(device)
+    link_ceiling = 3 * (1 << 30) / (e[0].elapsed_time(e[1]) * 1e-3) / 1e9
+    del hb, db
     out = {"workload": "weight restore: 57-block DiT, 1,140 bf16 tensors, 40 GiB pool, 2 MiB pages",
            "payload_bytes": int(wr.payload), "h2d_mode": h2d_mode,
            "h2d_put_ms": round(pm, 3), "h2d_link_gbs": round(wr.payload / (pm * 1e-3) / 1e9, 1),
+           "pinned_copy_ceiling_gbs": round(link_ceiling, 1),
+           "h2d_frac_of_pinned_copy": round(wr.payload / (pm * 1e-3) / 1e9 / link_ceiling, 3),
+           "h2d_vs_pcie_gen5_x16_64gbs": round(wr.payload / (pm * 1e-3) / 1e9 / 64.0, 2),
            "get_call_ms": round(gm, 3), "get_call_gbs": round(2 * wr.payload / (gm * 1e-3) / 1e9, 1),
            "get_kernel_ms": round(gk, 3), "get_gbs": round(2 * wr.payload / (gk * 1e-3) / 1e9, 1),
            "launches_per_rep": launches, "bit_exact": bool(ok)}

@@ -33,6 +33,7 @@
 #include <cstdint>
 #include <map>
 #include <memory>
+#include <mutex>
 #include <set>
 #include <string>
 #include <unordered_map>
@@ -219,5 +220,6 @@ class Control {
 // The opaque C handle around a control core.
 struct t2i_ctl {
     t2i::Control* core;
-    bool owned;      // false: borrowed from a store (queries only)
+    bool owned;                 // false: borrowed from a store (queries only)
+    std::mutex* mu = nullptr;   // the store's lock, for queries of a borrowed core
 };

@@ -16,12 +16,22 @@ const char* thread_error() { return g_thread_error.c_str(); }
 using t2i::Control;
 
 #define T2I_GUARD_BEGIN try {
-#define T2I_GUARD_END(ctl)                                     \
-    }                                                          \
-    catch (const std::bad_alloc&) {                            \
-        (ctl)->core->set_error("host memory allocation failed"); \
-        return T2I_ERR_INVALID;                                \
+#define T2I_GUARD_END(ctl)                                               \
+    }                                                                    \
+    catch (const std::exception& e) {                                    \
+        (ctl)->core->set_error(std::string("host error: ") + e.what());  \
+        return T2I_ERR_INVALID;                                          \
     }
+
+namespace {
+// Queries of a store's control core take the store's lock.
+struct QueryLock {
+    std::unique_lock<std::mutex> lk;
+    explicit QueryLock(const t2i_ctl* c) {
+        if (c->mu) lk = std::unique_lock<std::mutex>(*c->mu);
+    }
+};
+}  // namespace
 
 extern "C" {
 
@@ -36,10 +46,10 @@ t2i_status t2i_ctl_create(uint64_t total_pages, uint64_t page_bytes, uint32_t al
         return T2I_ERR_INVALID;
     }
     try {
-        t2i_ctl* c = new t2i_ctl{new Control(total_pages, page_bytes, alloc_policy), true};
+        t2i_ctl* c = new t2i_ctl{new Control(total_pages, page_bytes, alloc_policy), true, nullptr};
         *out = c;
-    } catch (const std::bad_alloc&) {
-        t2i::set_thread_error("t2i_ctl_create: host memory allocation failed");
+    } catch (const std::exception& e) {
+        t2i::set_thread_error(std::string("t2i_ctl_create: host error: ") + e.what());
         return T2I_ERR_INVALID;
     }
     return T2I_OK;
@@ -100,6 +110,7 @@ t2i_status t2i_ctl_compact(t2i_ctl* ctl, uint64_t limit_bytes, t2i_move* moves, 
 
 t2i_status t2i_ctl_object(const t2i_ctl* ctl, t2i_id id, t2i_object_info* info, uint32_t* pages, uint64_t cap) {
     if (!ctl) return T2I_ERR_INVALID;
+    QueryLock ql(ctl);
     const t2i::Object* o = ctl->core->find(id);
     if (!o) return ctl->core->is_evicted(id) ? T2I_ERR_EVICTED : T2I_ERR_NOT_FOUND;
     if (info) {
@@ -121,6 +132,7 @@ t2i_status t2i_ctl_object(const t2i_ctl* ctl, t2i_id id, t2i_object_info* info, 
 
 t2i_status t2i_ctl_free_pages(const t2i_ctl* ctl, uint32_t* out, uint64_t cap, uint64_t* n) {
     if (!ctl) return T2I_ERR_INVALID;
+    QueryLock ql(ctl);
     const std::vector<uint32_t> f = ctl->core->free_list();
     if (n) *n = f.size();
     if (out) {
@@ -132,6 +144,7 @@ t2i_status t2i_ctl_free_pages(const t2i_ctl* ctl, uint32_t* out, uint64_t cap, u
 
 t2i_status t2i_ctl_last_evictions(const t2i_ctl* ctl, t2i_id* out, uint64_t cap, uint64_t* n) {
     if (!ctl) return T2I_ERR_INVALID;
+    QueryLock ql(ctl);
     const auto& e = ctl->core->last_evictions();
     if (n) *n = e.size();
     if (out) {
@@ -143,6 +156,7 @@ t2i_status t2i_ctl_last_evictions(const t2i_ctl* ctl, t2i_id* out, uint64_t cap,
 
 t2i_status t2i_ctl_stats(const t2i_ctl* ctl, t2i_stats* out) {
     if (!ctl || !out) return T2I_ERR_INVALID;
+    QueryLock ql(ctl);
     ctl->core->stats(out);
     return T2I_OK;
 }

@@ -113,6 +113,7 @@ class Store {
           ctl_(cfg.pool_bytes / cfg.page_bytes, cfg.page_bytes, cfg.alloc_policy) {
         handle_.core = &ctl_;
         handle_.owned = false;
+        handle_.mu = &mu;
         page_shift_ = log2_exact(cfg.page_bytes);
     }
     ~Store() {
@@ -796,8 +797,8 @@ t2i_status t2i_store_create(void* pool_dev, const t2i_store_config* cfg, int dev
     Store* s = nullptr;
     try {
         s = new Store(pool_dev, *cfg, device);
-    } catch (const std::bad_alloc&) {
-        t2i::set_thread_error("t2i_store_create: host memory allocation failed");
+    } catch (const std::exception& e) {
+        t2i::set_thread_error(std::string("t2i_store_create: host error: ") + e.what());
         return T2I_ERR_INVALID;
     }
     std::string err;
@@ -818,6 +819,9 @@ t2i_status t2i_store_destroy(t2i_store* store) {
     return T2I_OK;
 }
 
+// Every store call: an NVTX range, the store's lock, and no C++ exception
+// past the C boundary (host memory exhaustion and the like become INVALID
+// with a message).
 #define T2I_STORE_CALL(store, expr)                                   \
     do {                                                              \
         if (!(store)) return T2I_ERR_INVALID;                         \
@@ -825,7 +829,8 @@ t2i_status t2i_store_destroy(t2i_store* store) {
         std::lock_guard<std::mutex> lock((store)->s->mu);             \
         try {                                                         \
             return (expr);                                            \
-        } catch (const std::bad_alloc&) {                             \
+        } catch (const std::exception& e) {                           \
+            (store)->s->set_error(std::string("host error: ") + e.what()); \
             return T2I_ERR_INVALID;                                   \
         }                                                             \
     } while (0)
@@ -871,7 +876,8 @@ t2i_status t2i_put_layers(t2i_store* store, const t2i_put_desc* descs, const uin
             try {
                 st = store->s->put(descs + layer_off[l], layer_off[l + 1] - layer_off[l], out_ids + layer_off[l],
                                    stream);
-            } catch (const std::bad_alloc&) {
+            } catch (const std::exception& e) {
+                store->s->set_error(std::string("host error: ") + e.what());
                 st = T2I_ERR_INVALID;
             }
         }
@@ -903,7 +909,8 @@ t2i_status t2i_pull(t2i_store* dst, t2i_store* src, const t2i_id* src_ids, uint3
     try {
         return dst->s->pull_from(*src->s, src_ids, n, consumers, out_ids, per_item,
                                  static_cast<cudaStream_t>(cuda_stream));
-    } catch (const std::bad_alloc&) {
+    } catch (const std::exception& e) {
+        dst->s->set_error(std::string("host error: ") + e.what());
         return T2I_ERR_INVALID;
     }
 }
