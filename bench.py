@@ -501,12 +501,13 @@ def time_weights(device, reps: int = 3, h2d_mode: int = 0):
 class Adapters:
     """Multi-tenant adapter cache: 512 LoRA sets (836 bf16 objects each) behind
     a 16 GiB pool of 256 KiB pages; each call gets a window of 256 objects of a
-    Zipf(1.1)-popular set. A set that is not resident (never loaded, or a
-    window object evicted) is put again from pinned host memory -- evicting
-    least recently used sets -- and the get is retried."""
+    Zipf(1.1)-popular set. Objects of a set that are not resident (never
+    loaded, or evicted: the last layers of the least recently used sets go
+    first, §5.3) are put again from pinned host memory before the get -- only
+    the missing ones, so a set's surviving first layers are reused."""
 
     def __init__(self, device, seed: int = 0, n_sets: int = 512, n_calls: int = 10_000,
-                 pool_bytes: int | None = None, window: int = 256):
+                 pool_bytes: int | None = None, window: int = 256, alloc_policy: int = 0):
         import torch
 
         from paper_2607_26566_gb300 import Store, get_descs, put_descs
@@ -530,28 +531,46 @@ class Adapters:
         self.off = W.lora_bank_offsets(seed, set_bytes, self.bank_bytes)
         self.sets, self.starts = W.adapter_calls(seed, n_calls, n_sets, 836, window, C_["zipf_s"])
         self.pool = torch.empty(pool_bytes or C_["pool_bytes"], dtype=torch.uint8, device=device)
-        self.store = Store(self.pool, C_["page_bytes"])
+        self.store = Store(self.pool, C_["page_bytes"], alloc_policy=alloc_policy)
         max_window = max(int(np.sort(v)[::-1][:window].sum()) for v in self.sizes.values())
         self.dst = torch.empty(max_window, dtype=torch.uint8, device=device)
-        self.ids = {}
+        self.ids = {}          # set -> ids of its objects (stale where evicted)
+        self.missing = {}      # set -> object indices evicted since their put
+        self.owner = {}        # live id -> (set, object index)
         self.loads = 0
         self.load_bytes = 0
+        self.load_objects = 0
+        self.window_misses = 0
         self.got_bytes = 0
         self.calls_done = 0
+        self.victims = []      # every eviction, in order (for comparison with the oracle)
 
     def load(self, s: int):
+        """Puts the missing objects of set s (all of them the first time)."""
         r = int(self.ranks[s])
-        old = self.ids.pop(s, None)
-        if old is not None:
-            self.store.check(self.store.free(old))
+        if s not in self.ids:
+            js = np.arange(len(self.sizes[r]))
+            self.ids[s] = np.zeros(len(js), np.uint64)
+        else:
+            js = np.array(sorted(self.missing.get(s, ())), np.int64)
+            if len(js) == 0:
+                return
         base = self.bank.data_ptr() + int(self.off[s])
-        d = self.put_descs(base + self.rel[r], nbytes=self.sizes[r], src_is_host=1, dtype_tag=W.DTYPE_BF16,
-                           group=s, order=self.blocks[r], evictable=1)
+        d = self.put_descs(base + self.rel[r][js], nbytes=self.sizes[r][js], src_is_host=1,
+                           dtype_tag=W.DTYPE_BF16, group=s, order=self.blocks[r][js], evictable=1)
         st, ids = self.store.put_batch(d)
         self.store.check(st)
-        self.ids[s] = ids
+        self.ids[s][js] = ids
+        self.missing[s] = set()
+        for j, i in zip(js, ids):
+            self.owner[int(i)] = (s, int(j))
+        for v in self.store.ctl.last_evictions():
+            s2, j2 = self.owner.pop(v)
+            self.missing.setdefault(s2, set()).add(j2)
+            self.victims.append(v)
         self.loads += 1
-        self.load_bytes += int(self.sizes[r].sum())
+        self.load_objects += len(js)
+        self.load_bytes += int(self.sizes[r][js].sum())
 
     def descs(self, k: int):
         s, w = int(self.sets[k]), int(self.starts[k])
@@ -561,15 +580,12 @@ class Adapters:
         return s, w, self.get_descs(self.ids[s][w:w + self.window], self.dst.data_ptr() + dst_rel, dst_bytes=sz)
 
     def call(self, k: int, stream=None):
-        s = int(self.sets[k])
-        if s not in self.ids:
+        s, w = int(self.sets[k]), int(self.starts[k])
+        if s not in self.ids or any(w <= j < w + self.window for j in self.missing.get(s, ())):
+            self.window_misses += 1
             self.load(s)
         s, w, d = self.descs(k)
         st, _ = self.store.get_batch(d, stream=stream, per_item=False)
-        if st == 4:  # EVICTED: reload the whole set and retry
-            self.load(s)
-            s, w, d = self.descs(k)
-            st, _ = self.store.get_batch(d, stream=stream, per_item=False)
         self.store.check(st)
         self.got_bytes += int(d["dst_bytes"].sum())
         self.calls_done += 1
@@ -641,8 +657,8 @@ def time_adapters(device, n_calls: int = 10_000, check_every: int = 500):
     out = {"workload": "adapters: 512 LoRA sets (ranks 8-64), 16 GiB pool, 256 KiB pages, Zipf(1.1), 256-object gets",
            "calls": n_calls, "ms": round(ms, 2), "calls_per_s": round(n_calls / (ms * 1e-3), 1),
            "wall_calls_per_s": round(n_calls / wall, 1),
-           "set_loads": ad.loads, "load_gib": round(ad.load_bytes / 2**30, 2),
-           "evictions": int(s1["evictions"] - s0["evictions"]), "misses": int(s1["misses"] - s0["misses"]),
+           "window_misses": ad.window_misses, "reloads": ad.loads, "reloaded_objects": ad.load_objects,
+           "load_gib": round(ad.load_bytes / 2**30, 2), "evictions": int(s1["evictions"] - s0["evictions"]),
            "all_calls_gbs": round((2 * ad.got_bytes + ad.load_bytes) / (ms * 1e-3) / 1e9, 1),
            "hit_calls": hit_calls, "hit_gbs": round(2 * hit_bytes / (hits_ms * 1e-3) / 1e9, 1),
            "hit_calls_per_s": round(hit_calls / (hits_ms * 1e-3), 1),
@@ -963,13 +979,10 @@ def time_views(device, adapter_calls: int = 3000):
     del wr
     torch.cuda.empty_cache()
     for policy in (0, 1):
-        ad = Adapters(device, n_calls=adapter_calls)
-        ad.store.close()
-        from paper_2607_26566_gb300 import Store
-        ad.store = Store(ad.pool, W.ADAPTERS["page_bytes"], alloc_policy=policy)
+        ad = Adapters(device, n_calls=adapter_calls, alloc_policy=policy)
         for k in range(adapter_calls):
             ad.call(k)
-        ids = [i for v in ad.ids.values() for i in v]
+        ids = list(ad.owner)
         frac, n = contiguous_fraction(ad.store, ids)
         out[f"adapters_policy{policy}_contiguous"] = round(frac, 4)
         out[f"adapters_policy{policy}_multipage_objects"] = n
