@@ -23,7 +23,7 @@ LIB = os.path.join(PKG, "libt2istore.so")
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 CXX_SOURCES = ["control.cpp", "ctl_capi.cpp", "prefix.cpp"]
 CU_SOURCES = ["store.cu"]
-HEADERS = ["control.hpp", "common.hpp", "deps.hpp", "kernels.cuh", "exports.map"]
+HEADERS = ["control.hpp", "common.hpp", "deps.hpp", "kernels.cuh", "launch.cuh", "exports.map"]
 
 
 def _cuda_home() -> str:
@@ -41,11 +41,12 @@ def _inputs() -> list[str]:
 
 
 def kernel_source_hash() -> str:
-    """Short hash of the device code and launch logic (ties profiles to a build)."""
+    """Short hash of the device code and the launch packing (ties profiles to
+    what a launch does)."""
     import hashlib
 
     h = hashlib.sha256()
-    for f in ("kernels.cuh", "store.cu", "deps.hpp"):
+    for f in ("kernels.cuh", "launch.cuh"):
         with open(os.path.join(CSRC, f), "rb") as fh:
             h.update(fh.read())
     return h.hexdigest()[:12]
