@@ -52,10 +52,10 @@ def parse():
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--no-cpu", action="store_true")
     p.add_argument("--no-extras", action="store_true", help="skip the one-call and reclaim variants")
-    p.add_argument("--sweep", action="store_true", help="also time B = 1 and B = 4")
+    p.add_argument("--no-sweep", action="store_true", help="skip timing B = 1 and B = 4")
     p.add_argument("--pool-gib", type=float, default=None, help="smaller pool (profiling small cases)")
     p.add_argument("--cpu-seconds", type=float, default=10.0, help="minimum CPU-baseline sample time")
-    p.add_argument("--rows", default="weights,adapters,compaction,prefix,views,pull",
+    p.add_argument("--rows", default="tiny,weights,adapters,compaction,prefix,views,pull",
                    help="other hot-path rows timed in the same run (comma list, or 'none')")
     p.add_argument("--adapter-calls", type=int, default=10_000)
     p.add_argument("--rows-only", action="store_true", help="skip the handoff headline (profiling a row)")
@@ -363,6 +363,57 @@ class Dist:
 def job_gbs(bytes_per_rank: float, ms_max: float, dist_ctx: "Dist") -> float:
     """Whole-job GB/s: the bytes every rank moved over the slowest rank's time."""
     return dist_ctx.sum(bytes_per_rank) / (ms_max * 1e-3) / 1e9
+
+
+# ----------------------------------------------------------------------------- tiny
+def time_tiny(device, reps: int = 20):
+    """The tiny store: 64 MiB pool, 64 KiB pages; put 32 objects (1 KiB - 2 MiB),
+    get all, free every third, put 8 more, get all 30 -- one step per rep."""
+    import torch
+
+    from paper_2607_26566_gb300 import Store, get_descs, put_descs
+
+    C_ = W.TINY
+    first, more = W.tiny_objects(0)
+    src1 = [torch.from_numpy(x).to(device) for x in first]
+    src2 = [torch.from_numpy(x).to(device) for x in more]
+    out1 = [torch.empty_like(x) for x in src1]
+    pool = torch.empty(C_["pool_bytes"], dtype=torch.uint8, device=device)
+    st = Store(pool, C_["page_bytes"])
+    gone_idx = W.tiny_freed_indices()
+    p1, p2 = put_descs(src1), put_descs(src2)
+    live_out = [o for k, o in enumerate(out1) if k not in gone_idx] + [torch.empty_like(x) for x in src2]
+    # put 32 + get 32 + put 8 + get 30: read + write bytes of each
+    payload = (2 * sum(x.numel() for x in src1) + 2 * sum(x.numel() for x in src2)
+               + 2 * sum(x.numel() for x in src1) + 2 * sum(o.numel() for o in live_out))
+
+    def step():
+        s, ids = st.put_batch(p1)
+        st.check(s)
+        st.check(st.get_batch(get_descs(ids, out1), per_item=False)[0])
+        st.check(st.free([int(ids[k]) for k in gone_idx]))
+        s, ids2 = st.put_batch(p2)
+        st.check(s)
+        keep = [int(ids[k]) for k in range(len(ids)) if k not in gone_idx] + [int(i) for i in ids2]
+        st.check(st.get_batch(get_descs(keep, live_out), per_item=False)[0])
+        st.check(st.free(keep))
+
+    stream = torch.cuda.current_stream(device)
+    for _ in range(3):
+        step()
+    torch.cuda.synchronize(device)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(reps):
+        step()
+    e1.record(stream)
+    torch.cuda.synchronize(device)
+    ms = e0.elapsed_time(e1) / reps
+    ok = all(torch.equal(a, b) for a, b in zip(out1, src1))
+    st.close()
+    return {"workload": "tiny: 64 MiB pool, 64 KiB pages, 32 + 8 uint8 objects (1 KiB - 2 MiB)",
+            "ms_per_step": round(ms, 4), "gbs": round(payload / (ms * 1e-3) / 1e9, 1), "bit_exact": bool(ok),
+            "launches_per_step": 4}
 
 
 # ----------------------------------------------------------------------------- weights
@@ -1142,6 +1193,8 @@ def run_reference(args, dist_ctx):
 def run_rows(args, device, peak):
     rows = {}
     wanted = [] if args.rows == "none" else [r.strip() for r in args.rows.split(",") if r.strip()]
+    if "tiny" in wanted:
+        rows["tiny"] = time_tiny(device)
     if "weights" in wanted:
         rows["weights"] = time_weights(device)
     if "adapters" in wanted:
@@ -1233,7 +1286,7 @@ def main():
         torch.cuda.empty_cache()
 
     sweep = {}
-    if args.sweep:
+    if not args.no_sweep:
         for Bs in (1, 4):
             hs = Handoff(Bs, args.requests, device)
             ms_s, _, _, _ = time_handoff(hs, max(3, args.steps // 2), args.warmup, dist_ctx, per_kernel=False)
