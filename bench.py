@@ -5,7 +5,10 @@ Workload (default): the T2I intermediate handoff -- 8 GiB pool of 2 MiB pages,
 bf16 pooled embeddings [B,768], fp32 latents [B,16,128,128] (got with the
 fused fp32 -> bf16 RNE cast) and fp16 decoded images [B,3,1024,1024]; B = 8.
 One step = put all 64 requests from producer buffers, get all 64 into consumer
-buffers, free everything: 128 batched calls, each one kernel launch.
+buffers, free everything: 128 batched calls, each one kernel launch. Request
+r is issued on stream r % 4 (--streams): independent requests overlap on the
+GPU, the store ordering each get after its own put and each reused page after
+its last reader.
 
 Metric: algorithmic read + write bytes / time (put and get: 2 x payload,
 cast get: 1.5 x the fp32 payload), GB/s, and its fraction of the measured
@@ -49,6 +52,7 @@ def parse():
     p.add_argument("--impl", default="native", choices=["native", "reference"])
     p.add_argument("--batch", type=int, default=8, help="B of the handoff workload")
     p.add_argument("--requests", type=int, default=64)
+    p.add_argument("--streams", type=int, default=4, help="streams the requests of a step are spread over")
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--no-cpu", action="store_true")
     p.add_argument("--no-extras", action="store_true", help="skip the one-call and reclaim variants")
@@ -231,6 +235,49 @@ class Handoff:
             if st:
                 raise RuntimeError("free: " + self.store.last_error())
 
+    def step_streams(self, streams, ev=None):
+        """One step with request r on ``streams[r % k]``: independent requests
+        overlap, so one launch's ramp and drain are hidden under another's
+        copy. The store orders each get after its request's put (same
+        stream) and each reused page after its last reader (page-level
+        events), so no further synchronisation is needed; the two phases
+        are still joined through ``streams[0]`` so that each phase's span is
+        measurable. ``ev`` = three timing events as in :meth:`step`."""
+        lib, h, n, k = self.lib, self.h, self.n_obj, len(streams)
+        ss = [C.c_void_p(x.cuda_stream) for x in streams]
+        if ev is not None:
+            ev[0].record(streams[0])
+        for r in range(self.requests):
+            st = lib.t2i_put_batch(h, self.pd_p[r], n, self.ids_p[r], ss[r % k])
+            if st:
+                raise RuntimeError("put_batch: " + self.store.last_error())
+        self._join(streams, ev[1] if ev is not None else None)
+        for r in range(self.requests):
+            self.gd[r]["id"] = self.ids[n * r:n * (r + 1)]
+            st = lib.t2i_get_batch(h, self.gd_p[r], n, None, ss[r % k])
+            if st:
+                raise RuntimeError("get_batch: " + self.store.last_error())
+        self._join(streams, ev[2] if ev is not None else None)
+        if not self.consumers:
+            st = lib.t2i_free(h, self.all_ids_p, len(self.ids))
+            if st:
+                raise RuntimeError("free: " + self.store.last_error())
+
+    def _join(self, streams, hub_event=None):
+        """Every stream waits until all of them reach this point (through
+        ``streams[0]``, where ``hub_event`` is recorded)."""
+        torch = self.torch
+        if not hasattr(self, "_done") or len(self._done) < len(streams):
+            self._done = [torch.cuda.Event() for _ in streams]
+            self._hub = torch.cuda.Event()
+        for x, e in zip(streams[1:], self._done):
+            e.record(x)
+            streams[0].wait_event(e)
+        hub = hub_event if hub_event is not None else self._hub
+        hub.record(streams[0])
+        for x in streams[1:]:
+            x.wait_event(hub)
+
     def step_two_streams(self, s_put, s_get):
         """The same step with puts on one stream and gets on another: the
         store orders each get after the put of its request only, so request
@@ -274,11 +321,24 @@ class Handoff:
                     raise RuntimeError("handoff output differs from its input")
 
 
-def time_handoff(hw: Handoff, steps: int, warmup: int, dist_ctx, per_kernel: bool, clocks_index=None):
+def time_handoff(hw: Handoff, steps: int, warmup: int, dist_ctx, per_kernel: bool, clocks_index=None,
+                 n_streams: int = 1):
+    """Times ``steps`` steps; with ``n_streams`` > 1 the requests of a step
+    are spread over that many streams (:meth:`Handoff.step_streams`).
+    ``per_kernel``: events around each phase (a run of one kernel's
+    launches); returns their mean spans and the bytes they moved."""
     torch = hw.torch
     stream = torch.cuda.current_stream(hw.device)
+    streams = [stream] + [torch.cuda.Stream(hw.device) for _ in range(n_streams - 1)]
+
+    def run(ev=None):
+        if n_streams == 1:
+            hw.step(stream.cuda_stream, ev)
+        else:
+            hw.step_streams(streams, ev)
+
     for _ in range(warmup):
-        hw.step(stream.cuda_stream)
+        run()
     torch.cuda.synchronize(hw.device)
     if per_kernel:
         # per step: the put phase and the get phase, each bracketed by events
@@ -296,9 +356,11 @@ def time_handoff(hw: Handoff, steps: int, warmup: int, dist_ctx, per_kernel: boo
     t1 = torch.cuda.Event(enable_timing=True)
     torch.cuda.nvtx.range_push("bench_timed")
     t0.record(stream)
+    for x in streams[1:]:
+        x.wait_event(t0)
     for k in range(steps):
-        hw.step(stream.cuda_stream, evs[k] if per_kernel else None)
-    t1.record(stream)
+        run(evs[k] if per_kernel else None)
+    t1.record(stream)        # every stream joined stream 0 at the end of the last step
     torch.cuda.nvtx.range_pop()
     torch.cuda.synchronize(hw.device)
     dist_ctx.barrier()
@@ -308,13 +370,12 @@ def time_handoff(hw: Handoff, steps: int, warmup: int, dist_ctx, per_kernel: boo
     launches = hw.store.stats()["launches"] - launches0
     kern = None
     if per_kernel:
-        # a phase holds hw.requests launches of its kernel
-        put_ms = [e[0].elapsed_time(e[1]) / hw.requests for e in evs]
-        get_ms = [e[1].elapsed_time(e[2]) / hw.requests for e in evs]
-        kern = {"put_ms": statistics.mean(put_ms), "get_ms": statistics.mean(get_ms),
-                "put_bytes": hw.put_bytes / hw.requests, "get_bytes": hw.get_bytes / hw.requests,
-                "put_total_ms": statistics.mean(put_ms) * hw.requests * steps,
-                "get_total_ms": statistics.mean(get_ms) * hw.requests * steps}
+        # a phase holds hw.requests launches of its kernel, n_streams at a time
+        put_ms = statistics.mean(e[0].elapsed_time(e[1]) for e in evs)
+        get_ms = statistics.mean(e[1].elapsed_time(e[2]) for e in evs)
+        kern = {"put_phase_ms": put_ms, "get_phase_ms": get_ms,
+                "put_phase_bytes": hw.put_bytes, "get_phase_bytes": hw.get_bytes,
+                "launches_per_phase": hw.requests, "streams": n_streams}
     return ms, launches, kern, (clk.summary() if clk else None)
 
 
@@ -1237,26 +1298,41 @@ def main():
     pool_bytes = int(args.pool_gib * (1 << 30)) if args.pool_gib else None
     hw = Handoff(B, args.requests, device, pool_bytes=pool_bytes)
     ms, launches, kern, clocks = time_handoff(hw, args.steps, args.warmup, dist_ctx, per_kernel=True,
-                                              clocks_index=dist_ctx.local)
+                                              clocks_index=dist_ctx.local, n_streams=args.streams)
     hw.verify()
     ms_max = dist_ctx.max(ms)
     value = job_gbs(hw.step_bytes * args.steps, ms_max, dist_ctx)
     peak, peak_kind = peaks()
 
-    # dominant kernel: the one with more total time in the timed region
-    dom = "gather_get_kernel" if kern["get_total_ms"] >= kern["put_total_ms"] else "scatter_put_kernel"
-    k_ms = kern["get_ms"] if dom == "gather_get_kernel" else kern["put_ms"]
-    k_bytes = kern["get_bytes"] if dom == "gather_get_kernel" else kern["put_bytes"]
-    achieved = k_bytes / (k_ms * 1e-3) / 1e9
+    def rates(kn):
+        return {"put": kn["put_phase_bytes"] / (kn["put_phase_ms"] * 1e-3) / 1e9,
+                "get": kn["get_phase_bytes"] / (kn["get_phase_ms"] * 1e-3) / 1e9}
+
+    # dominant kernel: the one with more time in the timed region; its phase
+    # (hw.requests launches, args.streams at a time) moves phase_bytes
+    dom = "gather_get_kernel" if kern["get_phase_ms"] >= kern["put_phase_ms"] else "scatter_put_kernel"
+    d, o = ("get", "put") if dom == "gather_get_kernel" else ("put", "get")
+    achieved = rates(kern)[d]
     traffic = ncu_traffic(dom, f"handoff_B{B}_request")
     roofline = {"bound": "hbm", "achieved": round(achieved, 1), "peak": peak, "unit": "GB/s",
                 "frac": round(achieved / peak, 4), "peak_kind": peak_kind,
                 "traffic": traffic,
-                "kernel": dom, "algorithmic_bytes_per_launch": k_bytes, "avg_launch_ms": round(k_ms, 5),
-                "other_kernel": {"name": "scatter_put_kernel" if dom == "gather_get_kernel" else "gather_get_kernel",
-                                 "achieved": round((kern["put_bytes"] / (kern["put_ms"] * 1e-3) / 1e9)
-                                                   if dom == "gather_get_kernel" else
-                                                   (kern["get_bytes"] / (kern["get_ms"] * 1e-3) / 1e9), 1)}}
+                "kernel": dom, "algorithmic_bytes_per_launch": kern[f"{d}_phase_bytes"] / hw.requests,
+                "launches_per_phase": hw.requests, "streams": args.streams,
+                "phase_ms": round(kern[f"{d}_phase_ms"], 5),
+                "achieved_is": "algorithmic bytes of the phase's launches / phase span (CUDA events)",
+                "other_kernel": {"name": "scatter_put_kernel" if d == "get" else "gather_get_kernel",
+                                 "achieved": round(rates(kern)[o], 1)}}
+    if args.streams > 1:
+        # the same workload on one stream: back-to-back launches, so the phase
+        # span / launches is each launch's own duration
+        ms1, _, kern1, _ = time_handoff(hw, max(3, args.steps // 2), args.warmup, dist_ctx, per_kernel=True)
+        r1 = rates(kern1)
+        roofline["one_stream"] = {"step_gbs": round(job_gbs(hw.step_bytes * max(3, args.steps // 2), dist_ctx.max(ms1),
+                                                            dist_ctx), 1),
+                                  "get_achieved": round(r1["get"], 1), "put_achieved": round(r1["put"], 1),
+                                  "get_frac": round(r1["get"] / peak, 4),
+                                  "get_avg_launch_ms": round(kern1["get_phase_ms"] / hw.requests, 5)}
     del hw
     torch.cuda.empty_cache()
 
@@ -1289,7 +1365,8 @@ def main():
     if not args.no_sweep:
         for Bs in (1, 4):
             hs = Handoff(Bs, args.requests, device)
-            ms_s, _, _, _ = time_handoff(hs, max(3, args.steps // 2), args.warmup, dist_ctx, per_kernel=False)
+            ms_s, _, _, _ = time_handoff(hs, max(3, args.steps // 2), args.warmup, dist_ctx, per_kernel=False,
+                                         n_streams=args.streams)
             sweep[f"B{Bs}"] = round(hs.step_bytes * max(3, args.steps // 2) / (ms_s * 1e-3) / 1e9, 1)
             del hs
             torch.cuda.empty_cache()
@@ -1298,8 +1375,10 @@ def main():
     if not args.no_e2e:
         he = Handoff(B, args.requests, device, host_buffers=True)
         e_steps = max(2, min(args.steps, 3))
-        ms_e, _, _, _ = time_handoff(he, e_steps, 1, dist_ctx, per_kernel=False)
+        ms_e, _, _, _ = time_handoff(he, e_steps, 3, dist_ctx, per_kernel=False, n_streams=args.streams)
         ms_e = dist_ctx.max(ms_e)
+        ms_e1, _, _, _ = time_handoff(he, e_steps, 1, dist_ctx, per_kernel=False)
+        ms_e1 = dist_ctx.max(ms_e1)
         # puts on one stream, gets on another: host-to-device and
         # device-to-host transfers overlap on the link
         s_put, s_get = torch.cuda.Stream(device), torch.cuda.Stream(device)
@@ -1318,7 +1397,9 @@ def main():
         e2e = {"value": round(job_gbs(he.step_bytes * e_steps, ms_e, dist_ctx), 2), "unit": "GB/s",
                "h2d_bytes_per_step": int(he.h2d_bytes), "d2h_bytes_per_step": int(he.d2h_bytes),
                "path": "t2i_put_batch / t2i_get_batch with pinned host sources and destinations",
-               "two_streams_value": round(job_gbs(he.step_bytes * e_steps, ms_e2, dist_ctx), 2)}
+               "streams": args.streams,
+               "one_stream_value": round(job_gbs(he.step_bytes * e_steps, ms_e1, dist_ctx), 2),
+               "puts_and_gets_on_two_streams_value": round(job_gbs(he.step_bytes * e_steps, ms_e2, dist_ctx), 2)}
         del he
         torch.cuda.empty_cache()
 
@@ -1338,6 +1419,7 @@ def main():
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "u8+f32->bf16",
             "data": "synthetic",
             "config": {"workload": f"t2i handoff, B={B}, {args.requests} requests in flight",
+                       "streams": args.streams,
                        "pool_bytes": pool_bytes or W.HANDOFF["pool_bytes"], "page_bytes": W.HANDOFF["page_bytes"],
                        "bytes_per_step": hw_bytes(B, args.requests), "l2": "inputs > L2 (no flush)",
                        "parallelism": f"replicas x{dist_ctx.world}"},

@@ -475,6 +475,60 @@ def test_independent_streams_do_not_wait_for_each_other():
     assert torch.equal(outs[0], x) and torch.equal(outs[1], y)
 
 
+def test_handoff_spread_over_streams():
+    """The handoff at B = 4 with request r on stream r % 4 and no
+    synchronisation between steps; steps alternate between two input sets and
+    two output sets, and one stream's gets of the first step run late, so a
+    put of the second step that reused a page before its last get read it
+    would show in the first step's outputs."""
+    C = W.HANDOFF
+    specs = W.handoff_specs(4)
+    n, R, k = len(specs), C["requests"], 4
+    st = make_store(C["pool_bytes"], C["page_bytes"])
+    streams = [torch.cuda.Stream() for _ in range(k)]
+    ins = [[W.handoff_request_torch(seed, r, specs, DEV) for r in range(R)] for seed in (0, 1)]
+    outs = [[[torch.empty_like(t) for t in ts] for ts in reqs] for reqs in ins]
+    torch.cuda.synchronize()
+    for rep in range(2):
+        for step in (0, 1):
+            ids = []
+            for r in range(R):
+                s, i = st.put_batch(put_descs(ins[step][r], nbytes=[sp.nbytes for sp in specs]),
+                                    stream=streams[r % k])
+                assert s == 0, st.last_error()
+                ids.append(i)
+            if step == 0:
+                _late(streams[1], 30)
+            for r in range(R):
+                s, _ = st.get_batch(get_descs(ids[r], outs[step][r]), stream=streams[r % k])
+                assert s == 0, st.last_error()
+            assert st.free(np.concatenate(ids)) == 0
+        torch.cuda.synchronize()
+        for step in (0, 1):
+            for r in range(R):
+                for j in range(n):
+                    assert torch.equal(outs[step][r][j], ins[step][r][j]), (rep, step, r, j)
+    assert st.stats()["used_pages"] == 0
+
+
+def test_bench_step_over_streams():
+    """The benchmark's own multi-stream step (phase joins included) gives
+    get(put(x)) == x and the oracle's cast at B = 1."""
+    import bench
+
+    hw = bench.Handoff(1, W.HANDOFF["requests"], DEV)
+    streams = [torch.cuda.current_stream()] + [torch.cuda.Stream() for _ in range(3)]
+    for _ in range(3):
+        hw.step_streams(streams)
+    torch.cuda.synchronize()
+    hw.verify()
+    for r in (0, 17, 63):
+        lat = hw.inputs[r][hw.ci].reshape(-1).view(torch.int32).cpu().numpy().view(np.uint32)
+        got = hw.outputs[r][hw.ci].view(torch.int16).cpu().numpy().view(np.uint16)
+        assert np.array_equal(got, f32_bits_to_bf16_bits(lat)), r
+    hw.store.close()
+
+
 def test_cross_stream_compaction():
     """A compaction on one stream waits for a late put of the pages it moves,
     and a get on a third stream waits for the compaction."""
