@@ -656,6 +656,7 @@ class Adapters:
         self.got_bytes = 0
         self.calls_done = 0
         self.victims = []      # every eviction, in order (for comparison with the oracle)
+        self.load_events = None  # a list: events around every reload put (timing)
 
     def load(self, s: int):
         """Puts the missing objects of set s (all of them the first time)."""
@@ -670,8 +671,14 @@ class Adapters:
         base = self.bank.data_ptr() + int(self.off[s])
         d = self.put_descs(base + self.rel[r][js], nbytes=self.sizes[r][js], src_is_host=1,
                            dtype_tag=W.DTYPE_BF16, group=s, order=self.blocks[r][js], evictable=1)
+        if self.load_events is not None:
+            ev = (self.torch.cuda.Event(enable_timing=True), self.torch.cuda.Event(enable_timing=True))
+            ev[0].record()
         st, ids = self.store.put_batch(d)
         self.store.check(st)
+        if self.load_events is not None:
+            ev[1].record()
+            self.load_events.append(ev)
         self.ids[s][js] = ids
         self.missing[s] = set()
         for j, i in zip(js, ids):
@@ -719,6 +726,7 @@ def time_adapters(device, n_calls: int = 10_000, check_every: int = 500):
     import torch
 
     ad = Adapters(device, n_calls=n_calls)
+    ad.load_events = []
     stream = torch.cuda.current_stream(device)
     torch.cuda.synchronize(device)
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
@@ -736,6 +744,7 @@ def time_adapters(device, n_calls: int = 10_000, check_every: int = 500):
     wall = time.perf_counter() - t_wall
     ms = e0.elapsed_time(e1)
     s1 = ad.store.stats()
+    load_ms = sum(a.elapsed_time(b) for a, b in ad.load_events)
     # the hit path alone: the same calls again with every set resident
     # (no misses are possible once a call's set has just been touched)
     hits_ms, hit_bytes, hit_calls = 0.0, 0, 0
@@ -771,6 +780,8 @@ def time_adapters(device, n_calls: int = 10_000, check_every: int = 500):
            "wall_calls_per_s": round(n_calls / wall, 1),
            "window_misses": ad.window_misses, "reloads": ad.loads, "reloaded_objects": ad.load_objects,
            "load_gib": round(ad.load_bytes / 2**30, 2), "evictions": int(s1["evictions"] - s0["evictions"]),
+           "miss_h2d_ms": round(load_ms, 2), "miss_h2d_link_gbs": round(ad.load_bytes / (load_ms * 1e-3) / 1e9, 1),
+           "miss_share_of_time": round(load_ms / ms, 4),
            "all_calls_gbs": round((2 * ad.got_bytes + ad.load_bytes) / (ms * 1e-3) / 1e9, 1),
            "hit_calls": hit_calls, "hit_gbs": round(2 * hit_bytes / (hits_ms * 1e-3) / 1e9, 1),
            "hit_calls_per_s": round(hit_calls / (hits_ms * 1e-3), 1),
@@ -1220,6 +1231,51 @@ def oracle_sample(B: int, n_requests: int, min_seconds: float = 0.0, max_steps: 
     return per_req * n_requests * steps / dt / 1e9, dt, per_req * n_requests * steps, steps
 
 
+def host_memcpy_sample(B: int, n_requests: int, min_seconds: float = 2.0, threads: int | None = None):
+    """A multithreaded host memcpy of the same step on the host cores: every
+    request's objects copied into 2 MiB pages of a host pool (put), then out
+    into consumer arrays (get, latents copied as fp32: no cast), split over
+    ``threads`` threads (numpy copies release the GIL). A reported baseline,
+    not the oracle. Returns (GB/s of 2 x copied bytes, seconds, threads)."""
+    from concurrent.futures import ThreadPoolExecutor
+
+    threads = threads or os.cpu_count() or 1
+    specs = W.handoff_specs(B)
+    P = W.HANDOFF["page_bytes"]
+    src = [np.random.default_rng(j).integers(0, 256, sp.nbytes, dtype=np.uint8) for j, sp in enumerate(specs)]
+    pages = sum(-(-sp.nbytes // P) for sp in specs)
+    pool = np.empty(n_requests * pages * P, np.uint8)
+    dst = [[np.empty(sp.nbytes, np.uint8) for sp in specs] for _ in range(n_requests)]
+    put, get = [], []
+    pg = 0
+    for r in range(n_requests):
+        for j, sp in enumerate(specs):
+            for o in range(0, sp.nbytes, P):
+                n = min(P, sp.nbytes - o)
+                put.append((pool[pg * P:pg * P + n], src[j][o:o + n]))
+                get.append((dst[r][j][o:o + n], pool[pg * P:pg * P + n]))
+                pg += 1
+    nbytes = 2 * sum(a.size for a, _ in put) * 2
+
+    def part(lst, i):
+        for a, b in lst[i::threads]:
+            np.copyto(a, b)
+
+    with ThreadPoolExecutor(threads) as ex:
+        for phase in (put, get):          # warm-up: touch every page
+            list(ex.map(lambda i: part(phase, i), range(threads)))
+        t = time.perf_counter()
+        steps = 0
+        while True:
+            for phase in (put, get):
+                list(ex.map(lambda i: part(phase, i), range(threads)))
+            steps += 1
+            dt = time.perf_counter() - t
+            if dt >= min_seconds:
+                break
+    return nbytes * steps / dt / 1e9, dt, threads
+
+
 # ----------------------------------------------------------------------------- main
 def run_reference(args, dist_ctx):
     if dist_ctx.rank != 0:
@@ -1411,6 +1467,10 @@ def main():
         cpu = {"value": round(v, 3), "unit": "GB/s", "cores": 1, "kind": "oracle",
                "sample": f"{n} full step(s) ({args.requests} B={B} requests put, got with the latents cast, "
                          f"freed) by the numpy oracle in {dt:.1f} s"}
+        mv, mdt, mthreads = host_memcpy_sample(B, 8)
+        cpu["host_memcpy"] = {"value": round(mv, 2), "unit": "GB/s", "cores": mthreads, "kind": "memcpy",
+                              "sample": f"8 B={B} requests copied into 2 MiB pages of a host pool and out "
+                                        f"again (no cast), {mthreads} threads, {mdt:.1f} s"}
 
     if dist_ctx.rank == 0:
         line = {

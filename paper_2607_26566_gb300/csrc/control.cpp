@@ -112,29 +112,6 @@ void FreePages::give(const std::vector<uint32_t>& pages, bool undo) {
     for (uint32_t p : pages) insert_page(p);
 }
 
-void FreePages::rebuild(uint64_t limit, const std::vector<uint8_t>& used) {
-    stack_.clear();
-    runs_.clear();
-    count_ = 0;
-    if (policy_ == 0) {
-        for (uint64_t p = limit; p-- > 0;)
-            if (!used[p]) stack_.push_back(static_cast<uint32_t>(p));
-        count_ = stack_.size();
-        return;
-    }
-    uint64_t p = 0;
-    while (p < limit) {
-        if (used[p]) {
-            ++p;
-            continue;
-        }
-        const uint64_t start = p;
-        while (p < limit && !used[p]) ++p;
-        runs_[uint32_t(start)] = uint32_t(p - start);
-        count_ += p - start;
-    }
-}
-
 std::vector<uint32_t> FreePages::list() const {
     if (policy_ == 0) return stack_;
     std::vector<uint32_t> out;
@@ -146,7 +123,23 @@ std::vector<uint32_t> FreePages::list() const {
 
 // ---------------------------------------------------------------- Control
 Control::Control(uint64_t total_pages, uint64_t page_bytes, uint32_t policy)
-    : P_(page_bytes), total_pages_(total_pages), limit_pages_(total_pages), free_(total_pages, policy) {}
+    : P_(page_bytes),
+      total_pages_(total_pages),
+      limit_pages_(total_pages),
+      free_(total_pages, policy),
+      page_obj_(total_pages, nullptr),
+      page_idx_(total_pages, 0) {}
+
+void Control::own(const Object* o) {
+    for (uint32_t j = 0; j < o->pages.size(); ++j) {
+        page_obj_[o->pages[j]] = const_cast<Object*>(o);
+        page_idx_[o->pages[j]] = j;
+    }
+}
+
+void Control::disown(const Object* o) {
+    for (uint32_t p : o->pages) page_obj_[p] = nullptr;
+}
 
 Control::~Control() {
     for (Object* o : live_) delete o;
@@ -188,6 +181,7 @@ void Control::flush_touches() {
 
 void Control::release(Object* o, bool evicted) {
     const uint64_t np = o->pages.size();
+    disown(o);
     free_.give(o->pages);
     used_pages_ -= np;
     Group* g = o->group;
@@ -215,8 +209,7 @@ void Control::release(Object* o, bool evicted) {
 
 uint64_t Control::live_pages_at_or_above(uint64_t limit) const {
     uint64_t k = 0;
-    for (const Object* o : live_)
-        for (uint32_t p : o->pages) k += p >= limit;
+    for (uint64_t p = limit; p < limit_pages_; ++p) k += page_obj_[p] != nullptr;
     return k;
 }
 
@@ -246,7 +239,12 @@ t2i_status Control::view(uint64_t id, const Object** out) {
 }
 
 void Control::rollback_compact() {
-    for (const Remap& r : last_remap_) r.o->pages[r.idx] = r.old_page;
+    for (const Remap& r : last_remap_) {
+        page_obj_[r.o->pages[r.idx]] = nullptr;
+        r.o->pages[r.idx] = r.old_page;
+        page_obj_[r.old_page] = r.o;
+        page_idx_[r.old_page] = r.idx;
+    }
     last_remap_.clear();
     free_.restore(std::move(last_free_));
     last_free_ = FreePages::Snapshot{};
@@ -330,6 +328,7 @@ t2i_status Control::put(const t2i_put_desc* descs, uint32_t n, t2i_id* ids, std:
         o->group = group_for(d.group);
         const uint64_t np = pages_for(d.nbytes);
         free_.take(np, &o->pages);
+        own(o);
         used_pages_ += np;
         Group* g = o->group;
         g->n_objects++;
@@ -360,6 +359,7 @@ void Control::rollback_put(const t2i_id* ids, uint32_t n) {
         counters_.puts--;
         counters_.bytes_put -= o->nbytes;
         const uint64_t np = o->pages.size();
+        disown(o);
         free_.give(o->pages, /*undo=*/true);
         used_pages_ -= np;
         Group* g = o->group;
@@ -482,6 +482,12 @@ t2i_status Control::free(const t2i_id* ids, uint32_t n) {
 }
 
 t2i_status Control::compact(uint64_t limit_bytes, std::vector<t2i_move>* moves) {
+    const t2i_status st = plan_compact(limit_bytes, moves);
+    if (st == T2I_OK) finish_compact();
+    return st;
+}
+
+t2i_status Control::plan_compact(uint64_t limit_bytes, std::vector<t2i_move>* moves) {
     moves->clear();
     if (limit_bytes % P_ != 0 || limit_bytes / P_ > total_pages_) {
         err_ = "compact: the limit must be a multiple of the page size and at most the pool";
@@ -492,46 +498,40 @@ t2i_status Control::compact(uint64_t limit_bytes, std::vector<t2i_move>* moves) 
         err_ = "compact: more pages are in use than the limit holds";
         return T2I_ERR_NOSPACE;
     }
-    struct Tail {
-        uint32_t page;
-        Object* o;
-        uint32_t idx;
-    };
-    std::vector<uint8_t> used(limit, 0);
-    std::vector<Tail> tail;
-    for (Object* o : live_) {
-        for (uint32_t j = 0; j < o->pages.size(); ++j) {
-            const uint32_t p = o->pages[j];
-            if (p < limit)
-                used[p] = 1;
-            else
-                tail.push_back({p, o, j});
-        }
-    }
-    std::sort(tail.begin(), tail.end(), [](const Tail& a, const Tail& b) { return a.page < b.page; });
-    moves->reserve(tail.size());
+    moves->reserve(live_pages_at_or_above(limit));
     last_remap_.clear();
-    last_remap_.reserve(tail.size());
+    last_remap_.reserve(moves->capacity());
     last_free_ = free_.snapshot();
     last_limit_ = limit_pages_;
     last_compact_counters_ = counters_;
+    // live pages at or above the limit, ascending (pages at or above the
+    // current limit are all free), each to the lowest free page below it
     uint64_t scan = 0;
     uint64_t moved_bytes = 0;
-    for (const Tail& t : tail) {
-        while (used[scan]) ++scan;  // used_pages_ <= limit guarantees a free page
+    for (uint64_t p = limit; p < limit_pages_; ++p) {
+        Object* o = page_obj_[p];
+        if (!o) continue;
+        while (page_obj_[scan]) ++scan;  // used_pages_ <= limit guarantees a free page
         const uint32_t dst = static_cast<uint32_t>(scan);
-        used[scan] = 1;
-        const uint64_t valid = std::min<uint64_t>(P_, t.o->nbytes - uint64_t(t.idx) * P_);
-        t.o->pages[t.idx] = dst;
-        last_remap_.push_back({t.o, t.idx, t.page});
-        moves->push_back({t.page, dst, valid});
+        const uint32_t idx = page_idx_[p];
+        const uint64_t valid = std::min<uint64_t>(P_, o->nbytes - uint64_t(idx) * P_);
+        o->pages[idx] = dst;
+        page_obj_[dst] = o;
+        page_idx_[dst] = idx;
+        page_obj_[p] = nullptr;
+        last_remap_.push_back({o, idx, static_cast<uint32_t>(p)});
+        moves->push_back({static_cast<uint32_t>(p), dst, valid});
         moved_bytes += valid;
     }
-    free_.rebuild(limit, used);
-    limit_pages_ = limit;
-    counters_.pages_moved += tail.size();
+    planned_limit_ = limit;
+    counters_.pages_moved += moves->size();
     counters_.bytes_moved += moved_bytes;
     return T2I_OK;
+}
+
+void Control::finish_compact() {
+    free_.rebuild(planned_limit_, [this](uint64_t q) { return page_obj_[q] != nullptr; });
+    limit_pages_ = planned_limit_;
 }
 
 void Control::stats(t2i_stats* out) const {

@@ -92,8 +92,30 @@ class FreePages {
         stack_ = std::move(s.stack);
         runs_ = std::move(s.runs);
     }
-    // after a compaction: every page below limit that `used` does not mark
-    void rebuild(uint64_t limit, const std::vector<uint8_t>& used);
+    // after a compaction: every page below limit for which used(p) is false
+    template <class Used>
+    void rebuild(uint64_t limit, Used used) {
+        stack_.clear();
+        runs_.clear();
+        count_ = 0;
+        if (policy_ == 0) {
+            for (uint64_t p = limit; p-- > 0;)
+                if (!used(p)) stack_.push_back(static_cast<uint32_t>(p));
+            count_ = stack_.size();
+            return;
+        }
+        uint64_t p = 0;
+        while (p < limit) {
+            if (used(p)) {
+                ++p;
+                continue;
+            }
+            const uint64_t start = p;
+            while (p < limit && !used(p)) ++p;
+            runs_.emplace_hint(runs_.end(), uint32_t(start), uint32_t(p - start));
+            count_ += p - start;
+        }
+    }
     // policy 0: the stack from bottom to top; policy 1: ascending
     std::vector<uint32_t> list() const;
 
@@ -160,6 +182,12 @@ class Control {
     t2i_status free(const t2i_id* ids, uint32_t n);
     // compact: plans, remaps and returns the moves (always filled).
     t2i_status compact(uint64_t limit_bytes, std::vector<t2i_move>* moves);
+    // The same in two halves, so that the free pages can be rebuilt while
+    // the moves run: plan_compact remaps and returns the moves;
+    // finish_compact (after a successful plan, before any other call)
+    // rebuilds the free pages and applies the new limit.
+    t2i_status plan_compact(uint64_t limit_bytes, std::vector<t2i_move>* moves);
+    void finish_compact();
     // Undo the last compaction (after a failed launch): page lists, the free
     // pages and the limit return to their state before it.
     void rollback_compact();
@@ -207,9 +235,17 @@ class Control {
         uint32_t idx;
         uint32_t old_page;
     };
+    // page -> (object, index in its page list); null for a free page. Kept
+    // on every put, release and move, so a compaction visits only the pages
+    // at or above its limit.
+    void own(const Object* o);
+    void disown(const Object* o);
+    std::vector<Object*> page_obj_;
+    std::vector<uint32_t> page_idx_;
     std::vector<Remap> last_remap_;          // the last compaction, for rollback_compact
     FreePages::Snapshot last_free_;
     uint64_t last_limit_ = 0;
+    uint64_t planned_limit_ = 0;
     t2i_stats last_compact_counters_{};
     t2i_stats counters_{};
     std::string err_;

@@ -343,6 +343,17 @@ t2i_status Store::put(const t2i_put_desc* descs, uint32_t n, t2i_id* ids, cudaSt
         ctl_.rollback_put(ids, n);
         return cuda_fail("put: cannot order after earlier calls", we);
     }
+    // The call's number goes on every page it writes once its copies are
+    // enqueued, and also when it fails part-way: copies enqueued before the
+    // failure may still be writing the pages it hands back.
+    auto mark_writes = [&]() {
+        uint32_t q = 0;
+        cudaError_t ee = deps_.end(&q);
+        for (uint32_t i = 0; i < n; ++i)
+            if (descs[i].src)
+                for (uint32_t pg : objs_[i]->pages) deps_.mark_write(pg, q);
+        return ee;
+    };
     segs_.clear();
     const uint64_t P = uint64_t(1) << page_shift_;
     for (uint32_t i = 0; i < n; ++i) {
@@ -361,6 +372,7 @@ t2i_status Store::put(const t2i_put_desc* descs, uint32_t n, t2i_id* ids, cudaSt
                                                 bytes, cudaMemcpyHostToDevice, stream);
                 if (e != cudaSuccess) {
                     err_ = std::string("put: host copy failed: ") + cudaGetErrorString(e);
+                    mark_writes();
                     ctl_.rollback_put(ids, n);
                     return T2I_ERR_CUDA;
                 }
@@ -374,15 +386,12 @@ t2i_status Store::put(const t2i_put_desc* descs, uint32_t n, t2i_id* ids, cudaSt
     if (!segs_.empty()) {
         st = launch_segments<Mode::Put>(segs_, stream);
         if (st != T2I_OK) {
+            mark_writes();
             ctl_.rollback_put(ids, n);
             return st;
         }
     }
-    uint32_t q = 0;
-    cudaError_t ee = deps_.end(&q);
-    for (uint32_t i = 0; i < n; ++i)
-        if (descs[i].src)
-            for (uint32_t pg : objs_[i]->pages) deps_.mark_write(pg, q);
+    cudaError_t ee = mark_writes();
     if (ee != cudaSuccess) return cuda_fail("put: cannot record its event", ee);
     return T2I_OK;
 }
@@ -459,11 +468,13 @@ t2i_status Store::get(const t2i_get_desc* descs, uint32_t n, t2i_status* per_ite
         cudaError_t we = deps_.wait();
         if (we != cudaSuccess) return cuda_fail("get: cannot order after earlier calls", we);
         st = launch_segments<Mode::Get>(segs_, stream);
-        if (st != T2I_OK) return st;  // nothing was counted: the get did not happen
+        // the pages carry this call as a reader even when it failed part-way
+        // (launches before the failure may still be reading them)
         uint32_t q = 0;
         cudaError_t ee = deps_.end(&q);
         for (const Seg& sg : segs_)
             for (uint32_t k = 0; k < sg.n_pages; ++k) deps_.mark_read(sg.pages[k], q);
+        if (st != T2I_OK) return st;  // nothing was counted: the get did not happen
         if (ee != cudaSuccess) st = cuda_fail("get: cannot record its event", ee);
     }
     // 3. LRU stamps and consumer counts, now that the copies are enqueued;
@@ -571,16 +582,18 @@ t2i_status Store::pull_from(Store& src, const t2i_id* ids, uint32_t n, uint32_t 
     }
     if (!segs_.empty()) {
         st = launch_segments<Mode::Move>(segs_, stream);
-        if (st != T2I_OK) {
-            ctl_.rollback_put(out_ids, n);  // the sources were not read: nothing counted
-            return st;
-        }
+        // marked even after a failure part-way: launches before it may still
+        // be reading the sources and writing the pages handed back
         uint32_t qd = 0, qs = 0;
         cudaError_t e1 = deps_.end(&qd);
         cudaError_t e2 = src.deps_.end(&qs);
         for (uint32_t i = 0; i < n; ++i) {
             for (uint32_t pg : objs_[i]->pages) deps_.mark_write(pg, qd);
             for (uint32_t pg : src_objs[i]->pages) src.deps_.mark_read(pg, qs);
+        }
+        if (st != T2I_OK) {
+            ctl_.rollback_put(out_ids, n);  // nothing counted on the sources
+            return st;
         }
         if (e1 != cudaSuccess || e2 != cudaSuccess)
             st = cuda_fail("pull: cannot record its event", e1 != cudaSuccess ? e1 : e2);
@@ -593,16 +606,23 @@ t2i_status Store::pull_from(Store& src, const t2i_id* ids, uint32_t n, uint32_t 
 
 t2i_status Store::compact(uint64_t limit_bytes, cudaStream_t stream, uint64_t* moved) {
     std::vector<t2i_move> moves;
-    t2i_status st = ctl_.compact(limit_bytes, &moves);
+    t2i_status st = ctl_.plan_compact(limit_bytes, &moves);
     if (moved) *moved = moves.size();
     if (st != T2I_OK) {
         err_ = ctl_.error();
         return st;
     }
-    if (moves.empty()) return T2I_OK;
+    if (moves.empty()) {
+        ctl_.finish_compact();
+        return T2I_OK;
+    }
     DeviceGuard g(device_);
     int si = 0;
-    if ((st = stream_slot(stream, &si)) != T2I_OK) return st;
+    if ((st = stream_slot(stream, &si)) != T2I_OK) {
+        ctl_.rollback_compact();
+        if (moved) *moved = 0;
+        return st;
+    }
     deps_.begin(si);
     for (const t2i_move& m : moves) {
         deps_.reads(m.src_page);
@@ -620,19 +640,22 @@ t2i_status Store::compact(uint64_t limit_bytes, cudaStream_t stream, uint64_t* m
     for (const t2i_move& m : moves)
         segs_.push_back({pool_ + uint64_t(m.src_page) * P, m.valid_bytes, &m.dst_page, 1u});
     st = launch_segments<Mode::Move>(segs_, stream);
-    if (st != T2I_OK) {
-        // the old pages still hold every byte: point the page tables back
-        ctl_.rollback_compact();
-        if (moved) *moved = 0;
-        return st;
-    }
+    // marked even after a failure part-way: moves launched before it may
+    // still be reading the old pages and writing the new ones
     uint32_t q = 0;
     cudaError_t ee = deps_.end(&q);
     for (const t2i_move& m : moves) {
         deps_.mark_read(m.src_page, q);
         deps_.mark_write(m.dst_page, q);
     }
-    if (st == T2I_OK && ee != cudaSuccess) st = cuda_fail("compact: cannot record its event", ee);
+    if (st != T2I_OK) {
+        // the old pages still hold every byte: point the page tables back
+        ctl_.rollback_compact();
+        if (moved) *moved = 0;
+        return st;
+    }
+    ctl_.finish_compact();  // the free pages are rebuilt while the moves run
+    if (ee != cudaSuccess) st = cuda_fail("compact: cannot record its event", ee);
     return st;
 }
 

@@ -107,3 +107,70 @@ def test_failed_pull_changes_neither_store():
     assert cons.get_batch(get_descs([int(j)], [out]))[0] == 0
     torch.cuda.synchronize()
     assert torch.equal(out, x)
+
+
+SLEEP_CYCLES_PER_MS = 2.0e6   # torch.cuda._sleep spins ~this many clock cycles per millisecond
+
+
+def _late(stream, ms):
+    """Keeps ``stream`` busy for about ``ms`` (torch's bounded sleep kernel)."""
+    with torch.cuda.stream(stream):
+        torch.cuda._sleep(int(ms * SLEEP_CYCLES_PER_MS))
+
+
+def test_failed_put_still_orders_the_pages_it_hands_back():
+    """A put that fails at its second launch has its first launch enqueued,
+    late, on its stream. The pages it hands back go to the next put, on
+    another stream, which must wait for that launch: else the late launch
+    overwrites the new object's bytes."""
+    P = 256
+    st = store(8000 * P, P)
+    s1, s2 = torch.cuda.Stream(), torch.cuda.Stream()
+    a = torch.randint(0, 256, (8000 * P,), dtype=torch.uint8, device=DEV)
+    b = torch.randint(0, 256, (8000 * P,), dtype=torch.uint8, device=DEV)
+    torch.cuda.synchronize()
+    _late(s1, 30)
+    assert st.inject_launch_failure(2) == 0          # 8,000 pages take two launches
+    s, _ = st.put_batch(put_descs([a]), stream=s1)
+    assert s == CUDA and st.stats()["used_pages"] == 0
+    s, (j,) = st.put_batch(put_descs([b]), stream=s2)
+    assert s == 0 and st.ctl.object(int(j))[2] == list(range(8000))   # the same pages
+    out = torch.zeros_like(b)
+    assert st.get_batch(get_descs([int(j)], [out]), stream=s2)[0] == 0
+    torch.cuda.synchronize()
+    assert torch.equal(out, b), "a launch of the failed put wrote pages handed to a later put"
+
+
+def test_failed_compaction_still_orders_the_pages_it_wrote():
+    """A compaction of 2,000 pages fails at its second launch, the first
+    (late on its stream) already enqueued. Its destination pages are free
+    again; a put on another stream that takes them must wait for that
+    launch. Every object, old and new, keeps its bytes."""
+    P = 4096
+    st = store(8000 * P, P)
+    s1, s2 = torch.cuda.Stream(), torch.cuda.Stream()
+    src = torch.randint(0, 256, (8000 * P,), dtype=torch.uint8, device=DEV)
+    new = torch.randint(0, 256, (2000 * P,), dtype=torch.uint8, device=DEV)
+    s, ids = st.put_batch(put_descs(src.data_ptr() + P * np.arange(8000), nbytes=np.full(8000, P)))
+    assert s == 0
+    assert st.free([int(i) for i in ids[0:4000:2]]) == 0      # pages 0, 2, ..., 3998
+    torch.cuda.synchronize()
+    _late(s1, 30)
+    assert st.inject_launch_failure(2) == 0
+    s, moved = st.compact(6000 * P, stream=s1)        # 2,000 one-page moves: two launches
+    assert s == CUDA and moved == 0
+    s, nids = st.put_batch(put_descs(new.data_ptr() + P * np.arange(2000), nbytes=np.full(2000, P)), stream=s2)
+    assert s == 0
+    assert sorted(p for i in nids for p in st.ctl.object(int(i))[2]) == list(range(0, 4000, 2))
+    out = torch.zeros(2000 * P, dtype=torch.uint8, device=DEV)
+    assert st.get_batch(get_descs(nids, out.data_ptr() + P * np.arange(2000), dst_bytes=np.full(2000, P)),
+                        stream=s2)[0] == 0
+    torch.cuda.synchronize()
+    assert torch.equal(out, new), "a launch of the failed compaction wrote pages handed to a later put"
+    live = [int(i) for i in ids[1:4000:2]] + [int(i) for i in ids[4000:]]
+    out = torch.zeros(len(live) * P, dtype=torch.uint8, device=DEV)
+    assert st.get_batch(get_descs(live, out.data_ptr() + P * np.arange(len(live)),
+                                  dst_bytes=np.full(len(live), P)))[0] == 0
+    torch.cuda.synchronize()
+    want = torch.cat([src[(2 * k + 1) * P:(2 * k + 2) * P] for k in range(2000)] + [src[4000 * P:]])
+    assert torch.equal(out, want)
