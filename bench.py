@@ -1276,6 +1276,71 @@ def host_memcpy_sample(B: int, n_requests: int, min_seconds: float = 2.0, thread
     return nbytes * steps / dt / 1e9, dt, threads
 
 
+def oracle_row_samples(rows: dict) -> None:
+    """The oracle as it stands, on a bounded sample of each row's workload
+    (single thread, the same byte counting as the row), added to the row as
+    ``cpu_oracle``. A reported baseline, not a target."""
+    from oracle import OK, OracleStore, PutItem
+
+    def entry(nbytes, dt, sample):
+        return {"value": round(nbytes / dt / 1e9, 3), "unit": "GB/s", "cores": 1, "kind": "oracle",
+                "sample": f"{sample}, {dt:.2f} s"}
+
+    if "weights" in rows:
+        specs = W.dit_weight_specs()
+        blk = [i for i, sp in enumerate(specs) if sp.block == 0]
+        g = np.random.default_rng(0)
+        data = [g.integers(0, 256, specs[i].nbytes, dtype=np.uint8) for i in blk]
+        ora = OracleStore(W.WEIGHTS["pool_bytes"], W.WEIGHTS["page_bytes"])
+        t = time.perf_counter()
+        st, ids = ora.put_batch([PutItem(d.size, d, W.DTYPE_BF16, 0, 0, True) for d in data])
+        st2, _, outs = ora.get_batch(ids)
+        dt = time.perf_counter() - t
+        assert st == OK and st2 == OK
+        n = sum(d.size for d in data)
+        rows["weights"]["cpu_oracle"] = entry(4 * n, dt, f"put + get of block 0 ({len(blk)} tensors, "
+                                                         f"{n / 2**20:.0f} MiB)")
+    if "adapters" in rows:
+        ranks = W.lora_ranks(0, 4)
+        ora = OracleStore(W.ADAPTERS["pool_bytes"], W.ADAPTERS["page_bytes"])
+        g = np.random.default_rng(0)
+        sets = []
+        for s_, r in enumerate(ranks):
+            objs = W.lora_objects(int(r))
+            st, ids = ora.put_batch([PutItem(nb, g.integers(0, 256, nb, dtype=np.uint8), W.DTYPE_BF16, s_, b, True)
+                                     for b, nb in objs])
+            assert st == OK
+            sets.append((ids, [nb for _, nb in objs]))
+        t = time.perf_counter()
+        nbytes = 0
+        for k in range(100):
+            ids, sz = sets[k % len(sets)]
+            w = (97 * k) % (len(ids) - 256)
+            st, _, _ = ora.get_batch(ids[w:w + 256])
+            assert st == OK
+            nbytes += 2 * sum(sz[w:w + 256])
+        rows["adapters"]["cpu_oracle"] = entry(nbytes, time.perf_counter() - t,
+                                               "100 hit gets of 256 objects over 4 resident sets")
+    if "compaction" in rows:
+        C_ = W.COMPACTION
+        pool = 4 << 30
+        P = C_["page_bytes"]
+        tr = W.compaction_trace(1, pool // P, P, 6250, C_["lo"], pool // 128, C_["p_free"], C_["settle_frac"])
+        ora = OracleStore(pool, P, keep_bytes=False, paged_pool=True)
+        ids = {}
+        for op in tr.ops:
+            if op[0] == "alloc":
+                ids[op[1]] = ora.put_batch([PutItem(op[2])])[1][0]
+            else:
+                ora.free([ids.pop(op[1])])
+        t = time.perf_counter()
+        st, moves = ora.compact(pool * 3 // 4)
+        dt = time.perf_counter() - t
+        assert st == OK
+        rows["compaction"]["cpu_oracle"] = entry(2 * sum(m[2] for m in moves), dt,
+                                                 f"compact of a 4 GiB paged pool to 3/4 ({len(moves)} pages moved)")
+
+
 # ----------------------------------------------------------------------------- main
 def run_reference(args, dist_ctx):
     if dist_ctx.rank != 0:
@@ -1460,6 +1525,8 @@ def main():
         torch.cuda.empty_cache()
 
     rows = run_rows(args, device, peak)
+    if not args.no_cpu and dist_ctx.rank == 0:
+        oracle_row_samples(rows)
 
     cpu = None
     if not args.no_cpu and dist_ctx.rank == 0:
