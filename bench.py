@@ -63,6 +63,8 @@ def parse():
                    help="other hot-path rows timed in the same run (comma list, or 'none')")
     p.add_argument("--adapter-calls", type=int, default=10_000)
     p.add_argument("--rows-only", action="store_true", help="skip the handoff headline (profiling a row)")
+    p.add_argument("--weight-blocks", type=int, default=None,
+                   help="restore only the first N blocks into a pool sized for them (profiling small cases)")
     p.add_argument("--compaction-gib", type=int, default=None,
                    help="smaller compaction pool (GiB; the limit is 3/4 of it): profiling small cases")
     return p.parse_args()
@@ -322,7 +324,7 @@ class Handoff:
 
 
 def time_handoff(hw: Handoff, steps: int, warmup: int, dist_ctx, per_kernel: bool, clocks_index=None,
-                 n_streams: int = 1):
+                 n_streams: int = 1, nvtx: str = "bench_timed"):
     """Times ``steps`` steps; with ``n_streams`` > 1 the requests of a step
     are spread over that many streams (:meth:`Handoff.step_streams`).
     ``per_kernel``: events around each phase (a run of one kernel's
@@ -354,7 +356,7 @@ def time_handoff(hw: Handoff, steps: int, warmup: int, dist_ctx, per_kernel: boo
     torch.cuda.synchronize(hw.device)
     t0 = torch.cuda.Event(enable_timing=True)
     t1 = torch.cuda.Event(enable_timing=True)
-    torch.cuda.nvtx.range_push("bench_timed")
+    torch.cuda.nvtx.range_push(nvtx)   # the headline's range is "bench_timed" (profiles filter on it)
     t0.record(stream)
     for x in streams[1:]:
         x.wait_event(t0)
@@ -485,7 +487,7 @@ class WeightRestore:
     contiguous per-block buffers (each tensor 256-byte aligned in its block)."""
 
     def __init__(self, device, seed: int = 0, h2d_mode: int = 0, n_blocks: int | None = None,
-                 alloc_policy: int = 0):
+                 alloc_policy: int = 0, pool_bytes: int | None = None):
         import torch
 
         from paper_2607_26566_gb300 import Store, get_descs, put_descs
@@ -498,7 +500,11 @@ class WeightRestore:
         if n_blocks is not None:
             layout = layout[:n_blocks]
         self.specs, self.layout = specs, layout
-        self.pool = torch.empty(C_["pool_bytes"], dtype=torch.uint8, device=device)
+        if pool_bytes is None and n_blocks is not None:
+            # room for the blocks' pages (each tensor rounded up to whole pages)
+            P = C_["page_bytes"]
+            pool_bytes = sum(-(-specs[i].nbytes // P) * P for _, members in layout for i, _ in members)
+        self.pool = torch.empty(pool_bytes or C_["pool_bytes"], dtype=torch.uint8, device=device)
         self.store = Store(self.pool, C_["page_bytes"], h2d_mode=h2d_mode, alloc_policy=alloc_policy)
         self.host = []      # pinned per-block source buffers
         self.dst = []       # device per-block destination buffers
@@ -551,10 +557,10 @@ class WeightRestore:
         self.store.close()
 
 
-def time_weights(device, reps: int = 3, h2d_mode: int = 0):
+def time_weights(device, reps: int = 3, h2d_mode: int = 0, n_blocks: int | None = None):
     import torch
 
-    wr = WeightRestore(device, h2d_mode=h2d_mode)
+    wr = WeightRestore(device, h2d_mode=h2d_mode, n_blocks=n_blocks)
     stream = torch.cuda.current_stream(device)
     wr.put_all()
     wr.get_all()
@@ -594,7 +600,8 @@ def time_weights(device, reps: int = 3, h2d_mode: int = 0):
     torch.cuda.synchronize(device)
     link_ceiling = 3 * (1 << 30) / (e[0].elapsed_time(e[1]) * 1e-3) / 1e9
     del hb, db
-    out = {"workload": "weight restore: 57-block DiT, 1,140 bf16 tensors, 40 GiB pool, 2 MiB pages",
+    out = {"workload": ("weight restore: 57-block DiT, 1,140 bf16 tensors, 40 GiB pool, 2 MiB pages" if n_blocks is None
+                        else f"weight restore (small case): the first {n_blocks} blocks, {wr.n_tensors} tensors"),
            "payload_bytes": int(wr.payload), "h2d_mode": h2d_mode,
            "h2d_put_ms": round(pm, 3), "h2d_link_gbs": round(wr.payload / (pm * 1e-3) / 1e9, 1),
            "pinned_copy_ceiling_gbs": round(link_ceiling, 1),
@@ -1378,7 +1385,7 @@ def run_rows(args, device, peak):
     if "tiny" in wanted:
         rows["tiny"] = time_tiny(device)
     if "weights" in wanted:
-        rows["weights"] = time_weights(device)
+        rows["weights"] = time_weights(device, n_blocks=args.weight_blocks)
     if "adapters" in wanted:
         rows["adapters"] = time_adapters(device, n_calls=args.adapter_calls)
     if "compaction" in wanted:
@@ -1447,7 +1454,8 @@ def main():
     if args.streams > 1:
         # the same workload on one stream: back-to-back launches, so the phase
         # span / launches is each launch's own duration
-        ms1, _, kern1, _ = time_handoff(hw, max(3, args.steps // 2), args.warmup, dist_ctx, per_kernel=True)
+        ms1, _, kern1, _ = time_handoff(hw, max(3, args.steps // 2), args.warmup, dist_ctx, per_kernel=True,
+                                        nvtx="bench_one_stream")
         r1 = rates(kern1)
         roofline["one_stream"] = {"step_gbs": round(job_gbs(hw.step_bytes * max(3, args.steps // 2), dist_ctx.max(ms1),
                                                             dist_ctx), 1),
@@ -1475,7 +1483,7 @@ def main():
         hx.store.close()
         del hx
         hr = Handoff(B, args.requests, device, pool_bytes=pool_bytes, consumers=1)
-        ms_r, _, _, _ = time_handoff(hr, 10, 3, dist_ctx, per_kernel=False)
+        ms_r, _, _, _ = time_handoff(hr, 10, 3, dist_ctx, per_kernel=False, nvtx="bench_reclaim")
         extras["reclaim_by_consumers_gbs"] = round(hr.step_bytes * 10 / (ms_r * 1e-3) / 1e9, 1)
         extras["reclaimed_per_step"] = hr.store.stats()["reclaimed"] // 13
         hr.store.close()
@@ -1487,7 +1495,7 @@ def main():
         for Bs in (1, 4):
             hs = Handoff(Bs, args.requests, device)
             ms_s, _, _, _ = time_handoff(hs, max(3, args.steps // 2), args.warmup, dist_ctx, per_kernel=False,
-                                         n_streams=args.streams)
+                                         n_streams=args.streams, nvtx="bench_sweep")
             sweep[f"B{Bs}"] = round(hs.step_bytes * max(3, args.steps // 2) / (ms_s * 1e-3) / 1e9, 1)
             del hs
             torch.cuda.empty_cache()
@@ -1496,9 +1504,10 @@ def main():
     if not args.no_e2e:
         he = Handoff(B, args.requests, device, host_buffers=True)
         e_steps = max(2, min(args.steps, 3))
-        ms_e, _, _, _ = time_handoff(he, e_steps, 3, dist_ctx, per_kernel=False, n_streams=args.streams)
+        ms_e, _, _, _ = time_handoff(he, e_steps, 3, dist_ctx, per_kernel=False, n_streams=args.streams,
+                                     nvtx="bench_e2e")
         ms_e = dist_ctx.max(ms_e)
-        ms_e1, _, _, _ = time_handoff(he, e_steps, 1, dist_ctx, per_kernel=False)
+        ms_e1, _, _, _ = time_handoff(he, e_steps, 1, dist_ctx, per_kernel=False, nvtx="bench_e2e")
         ms_e1 = dist_ctx.max(ms_e1)
         # puts on one stream, gets on another: host-to-device and
         # device-to-host transfers overlap on the link

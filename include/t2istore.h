@@ -146,13 +146,17 @@ typedef struct t2i_object_info {
 
 /* Creates a store over [pool_dev, pool_dev + pool_bytes) on CUDA device
  * `device`. pool_dev must be device memory of that device, 256-byte aligned.
- * The store never frees pool_dev. Errors: INVALID (geometry, pointer),
- * CUDA (device query failed). On error *out is NULL and t2i_last_error(NULL)
- * describes it.                                                             */
+ * The store never frees pool_dev. It allocates 2 KiB of device memory of its
+ * own (cudaMalloc, cleared on a private stream before this returns): the
+ * chunk counters through which the CTAs of a large launch share out its
+ * work, one for each of the first 64 streams the store is given (launches
+ * on later streams split their work statically). t2i_store_destroy frees it.
+ * Errors: INVALID (geometry, pointer), CUDA (device query or allocation
+ * failed). On error *out is NULL and t2i_last_error(NULL) describes it.     */
 t2i_status t2i_store_create(void* pool_dev, const t2i_store_config* cfg, int device, t2i_store** out);
 
-/* Frees the store's host state and events after waiting for the work of
- * every stream it was given.
+/* Frees the store's host state, events and chunk counters after waiting for
+ * the work of every stream it was given.
  * Does not free the pool. NULL is accepted.                                 */
 t2i_status t2i_store_destroy(t2i_store* store);
 

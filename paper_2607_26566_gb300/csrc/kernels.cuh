@@ -2,13 +2,19 @@
 // (put), gather (get), gather with a fused fp32 -> bf16 round-to-nearest-even
 // cast, and live-page moves (compaction). All four are one copy engine. A
 // launch carries its descriptors in its own parameter space (up to ~31 KiB):
-// no device scratch memory and no host->device descriptor copy.
+// no host->device descriptor copy.
 //
 // Work split: the segments of a launch are laid end to end in a "launch byte
-// space" (each starting on a 32-byte granule) and every CTA takes an equal,
-// contiguous share of it, so all CTAs finish together. A CTA walks its share
-// in pieces of at most U = 32 KiB that lie in one page of one segment,
-// mapping each piece to its page through the segment's page list.
+// space" (each starting on a 32-byte granule). In a large launch (>= 1 MiB
+// per resident CTA) CTAs take 32 KiB chunks of it one at a time from a
+// counter in device memory (the store's work counter for the launch's
+// stream), so CTAs on SMs that get more bandwidth take more chunks and all
+// CTAs finish within about one chunk of each other: with equal static shares
+// the last CTAs of a large launch finished ~1.6x later than the first on
+// GB300. Smaller launches (work == 0) give each CTA an equal contiguous
+// share. A CTA walks its part in pieces of at most U = 32 KiB that lie in
+// one page of one segment, mapping each piece to its page through the
+// segment's page list.
 //
 // HBM-bound by construction (2 bytes of traffic per payload byte, 1.5 for the
 // cast): fully coalesced 16-byte accesses, enough bytes in flight per SM (8
@@ -62,15 +68,41 @@ static_assert(sizeof(SegDesc) == 24, "SegDesc layout");
 constexpr uint64_t kCastFlag = uint64_t(1) << 63;
 
 struct LaunchHeader {
-    uint64_t pool;          // pool base address (device)
+    uint64_t pool;            // pool base address (device)
+    uint64_t work;            // device address of the launch's WorkCounter; 0 = equal static shares
     uint32_t n_seg;
-    uint32_t n_granules;    // size of the launch byte space in granules
+    uint32_t n_granules;      // size of the launch byte space in granules
     uint32_t page_shift;
-    uint32_t piece_bytes;   // min(U, page size)
-    uint32_t pages_offset;  // byte offset of the uint32 page array in blob
-    uint32_t pad;
+    uint32_t piece_bytes;     // min(U, page size)
+    uint32_t pages_offset;    // byte offset of the uint32 page array in blob
+    uint32_t chunk_granules;  // granules a CTA takes at a time from the counter
+    uint32_t pad[2];
 };
-static_assert(sizeof(LaunchHeader) == 32, "LaunchHeader layout");
+static_assert(sizeof(LaunchHeader) == 48, "LaunchHeader layout");
+
+// The chunk counter of one stream of a store. Zero between launches: the
+// last CTA of every launch that used it puts both fields back to zero, and
+// the next launch on the same stream reads it only after that launch has
+// completed (griddepcontrol.wait, or plain stream order).
+struct WorkCounter {
+    unsigned int next;  // chunks handed out
+    unsigned int done;  // CTAs finished
+    unsigned int pad[6];
+};
+static_assert(sizeof(WorkCounter) == 32, "WorkCounter layout");
+#ifndef T2I_TUNE_CHUNK_GRANULES
+#define T2I_TUNE_CHUNK_GRANULES 1024
+#endif
+#ifndef T2I_TUNE_DYN_MIN_CTA_BYTES
+#define T2I_TUNE_DYN_MIN_CTA_BYTES (1ull << 20)
+#endif
+// 32 KiB chunks (a sweep: 16 and 64 KiB were slower on large launches)
+constexpr uint32_t kChunkGranules = T2I_TUNE_CHUNK_GRANULES;
+// Launches with fewer bytes per resident CTA than this use equal static
+// shares: there the barrier each chunk costs more than the imbalance it
+// removes (a sweep: a B=8 handoff request, 395 KiB per CTA, and 256-object
+// adapter gets lost up to 5% with chunks; 0.7-3 GiB launches gained 6-12%).
+constexpr uint64_t kDynMinCtaBytes = T2I_TUNE_DYN_MIN_CTA_BYTES;
 
 template <int BLOB>
 struct LaunchParams {
@@ -301,7 +333,53 @@ __device__ __forceinline__ void pdl_wait_then_release() {
 // small enough for kMinBlocks resident CTAs per SM. GENERAL = true adds the
 // shifted copies and the element-wise cast for any alignment.
 template <Mode M, bool GENERAL, int BLOB>
+__device__ __forceinline__ void run_range(const LaunchParams<BLOB>& p, uint64_t g0, uint64_t g1);
+
+// This CTA's part of the launch: chunks from the counter, or an equal share.
+template <Mode M, bool GENERAL, int BLOB>
 __device__ __forceinline__ void run_share(const LaunchParams<BLOB>& p) {
+    if (p.h.work == 0) {
+        const uint64_t g0 = uint64_t(p.h.n_granules) * blockIdx.x / gridDim.x;
+        const uint64_t g1 = uint64_t(p.h.n_granules) * (blockIdx.x + 1) / gridDim.x;
+        run_range<M, GENERAL, BLOB>(p, g0, g1);
+        return;
+    }
+    // (the counter's address and the sizes are re-read from the parameters
+    // where needed: they take no registers across the copy)
+    // Two ticket slots: the ticket for chunk k+1 is written into the slot
+    // not read in round k, so one barrier per chunk suffices.
+    __shared__ uint32_t s_next[2];
+    if (threadIdx.x == 0) s_next[0] = atomicAdd(&reinterpret_cast<WorkCounter*>(p.h.work)->next, 1u);
+    __syncthreads();
+    uint32_t c = s_next[0];
+    uint32_t k = 0;
+#pragma unroll 1
+    while (uint64_t(c) * p.h.chunk_granules < p.h.n_granules) {
+        // the next chunk is fetched while this one is copied
+        uint32_t t = 0;
+        if (threadIdx.x == 0) t = atomicAdd(&reinterpret_cast<WorkCounter*>(p.h.work)->next, 1u);
+        const uint64_t g0 = uint64_t(c) * p.h.chunk_granules;
+        run_range<M, GENERAL, BLOB>(p, g0, umin64(g0 + p.h.chunk_granules, p.h.n_granules));
+        k ^= 1u;
+        if (threadIdx.x == 0) s_next[k] = t;
+        __syncthreads();
+        c = s_next[k];
+    }
+    // the last CTA out leaves the counter at zero for the next launch
+    if (threadIdx.x == 0) {
+        WorkCounter* wc = reinterpret_cast<WorkCounter*>(p.h.work);
+        __threadfence();
+        if (atomicAdd(&wc->done, 1u) == gridDim.x - 1) {
+            wc->next = 0;
+            wc->done = 0;
+            __threadfence();
+        }
+    }
+}
+
+// Copies granules [g0, g1) of the launch byte space.
+template <Mode M, bool GENERAL, int BLOB>
+__device__ __forceinline__ void run_range(const LaunchParams<BLOB>& p, uint64_t g0, uint64_t g1) {
     // the general kernels run at 2 CTAs/SM with room for the shifted paths:
     // they take half the vectors per round (a piece is then two rounds)
     constexpr int kV = GENERAL ? kVecPerThread / 2 : kVecPerThread;
@@ -311,9 +389,6 @@ __device__ __forceinline__ void run_share(const LaunchParams<BLOB>& p) {
     const uint32_t pshift = p.h.page_shift;
     const uint64_t pmask = (uint64_t(1) << pshift) - 1;
     const uint64_t piece = p.h.piece_bytes;
-    // this CTA's share of the launch byte space, in whole granules
-    const uint64_t g0 = uint64_t(p.h.n_granules) * blockIdx.x / gridDim.x;
-    const uint64_t g1 = uint64_t(p.h.n_granules) * (blockIdx.x + 1) / gridDim.x;
     if (g0 == g1) return;
     uint64_t pos = g0 * kGranule;
     const uint64_t end = g1 * kGranule;

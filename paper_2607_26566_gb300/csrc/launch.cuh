@@ -13,12 +13,16 @@ t2i_status Store::launch_one(const std::vector<SegDesc>& sd, const std::vector<u
                              cudaStream_t stream) {
     auto* p = reinterpret_cast<LaunchParams<BLOB>*>(param_buf_);
     p->h.pool = pool_;
+    p->h.work = uint64_t(n_granules) * kGranule >= kDynMinCtaBytes * uint64_t(max_ctas_[int(M)][GENERAL ? 1 : 0])
+                    ? cur_work_
+                    : 0;
+    p->h.chunk_granules = kChunkGranules;
+    p->h.pad[0] = p->h.pad[1] = 0;
     p->h.n_seg = static_cast<uint32_t>(sd.size());
     p->h.n_granules = n_granules;
     p->h.page_shift = page_shift_;
     p->h.piece_bytes = static_cast<uint32_t>(std::min<uint64_t>(kPieceBytes, uint64_t(1) << page_shift_));
     p->h.pages_offset = static_cast<uint32_t>(sd.size() * sizeof(SegDesc));
-    p->h.pad = 0;
     std::memcpy(p->blob, sd.data(), sd.size() * sizeof(SegDesc));
     std::memcpy(p->blob + p->h.pages_offset, pages.data(), pages.size() * sizeof(uint32_t));
     // every CTA gets at least kMinCtaBytes of the launch (small batches use a

@@ -120,6 +120,7 @@ class Store {
         DeviceGuard g(device_);
         deps_.synchronize_all();
         deps_.release();
+        if (work_) cudaFree(work_);
     }
 
     t2i_status init(std::string* err) {
@@ -143,6 +144,23 @@ class Store {
                 cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, fns[m][g], kThreads, 0);
                 max_ctas_[m][g] = sms * (occ > 0 ? occ : 1);
             }
+        // one chunk counter per stream (the first kWorkStreams streams of
+        // the store; later ones use equal static shares), zeroed once
+        if (cudaMalloc(&work_, kWorkStreams * sizeof(WorkCounter)) != cudaSuccess) {
+            work_ = nullptr;
+            *err = "cannot allocate the work counters";
+            return T2I_ERR_CUDA;
+        }
+        // cleared on a private non-blocking stream: waits for nothing else
+        cudaStream_t zs = nullptr;
+        bool zeroed = cudaStreamCreateWithFlags(&zs, cudaStreamNonBlocking) == cudaSuccess &&
+                      cudaMemsetAsync(work_, 0, kWorkStreams * sizeof(WorkCounter), zs) == cudaSuccess &&
+                      cudaStreamSynchronize(zs) == cudaSuccess;
+        if (zs) cudaStreamDestroy(zs);
+        if (!zeroed) {
+            *err = "cannot clear the work counters";
+            return T2I_ERR_CUDA;
+        }
         deps_.resize_pages(ctl_.total_pages());
         return T2I_OK;
     }
@@ -190,13 +208,16 @@ class Store {
     template <Mode M, bool GENERAL, int BLOB>
     t2i_status launch_one(const std::vector<SegDesc>& sd, const std::vector<uint32_t>& pages, uint32_t n_granules,
                           cudaStream_t stream);
-    // the call's stream in the dependency tracker (creating its events)
+    // the call's stream in the dependency tracker (creating its events), and
+    // the work counter its launches use
     t2i_status stream_slot(cudaStream_t s, int* si) {
         *si = deps_.stream_index(s);
         if (*si < 0) {
             err_ = "cannot create the events for a new stream";
             return T2I_ERR_CUDA;
         }
+        cur_work_ = *si < int(kWorkStreams) ? reinterpret_cast<uint64_t>(work_) + uint64_t(*si) * sizeof(WorkCounter)
+                                             : 0;
         return T2I_OK;
     }
     t2i_status cuda_fail(const char* what, cudaError_t e) {
@@ -212,6 +233,12 @@ class Store {
     uint32_t page_shift_ = 0;
     int max_ctas_[3][2] = {{1, 1}, {1, 1}, {1, 1}};  // [mode][any alignment]: resident CTAs on the device
     uint32_t fail_countdown_ = 0;  // > 0: that many launches from now, report a failure (testing)
+    // Work counters, one per stream index: launches on one stream run one
+    // after another (each waits for the previous grid before touching its
+    // counter), launches on different streams use different counters.
+    static constexpr uint32_t kWorkStreams = 64;
+    WorkCounter* work_ = nullptr;
+    uint64_t cur_work_ = 0;  // the current call's counter (0: static shares)
     std::vector<Seg> aligned_, general_;
     StreamDeps deps_;
     std::string err_;
