@@ -288,6 +288,53 @@ const char* t2i_ctl_last_error(const t2i_ctl* ctl);
 t2i_status t2i_inject_launch_failure(t2i_store* store, uint32_t countdown);
 
 /* =========================================================================
+ * Gather without allocation. The paper has no counterpart: this is an extra
+ * entry point of the library, not a step of the method.
+ * ========================================================================= */
+
+/* Copies one object's pages out of a pool into a contiguous device buffer,
+ * as a one-item t2i_get_batch does (the same gather kernel, the same bytes,
+ * the same optional fp32 -> bf16 RNE cast), but with no store and without
+ * allocating any memory.
+ *
+ * Who needs it: a caller that must not allocate device memory while it
+ * moves data. In a serving process the free HBM is often reserved up front
+ * (by the inference engine, or by PyTorch's caching allocator), so a new
+ * cudaMalloc there fails, and a cudaFree waits for the whole device. Code
+ * that holds a pool and its page lists but no t2i_store is in the same
+ * position: a store allocates its chunk counters when it is created.
+ *
+ * Scratch: the CTAs of a launch take their chunks from counters kept in a
+ * static 2 KiB device array of the library (64 counters of 32 bytes: one
+ * per launch of a call). Every GPU that loads the library holds the array
+ * until the process exits. A call first zeroes the counters it will use
+ * (cudaMemsetAsync on cuda_stream), because every call shares the array and
+ * it keeps whatever the last call left. Calls that overlap on the GPU (on
+ * other streams or from other threads) race on the counters and can skip or
+ * repeat chunks: order such calls on one stream. The first call on a device
+ * sets up that device: it looks up the array's device address
+ * (cudaGetSymbolAddress) and the gather kernels' occupancy. Make that first
+ * call before any stream capture. No call allocates: no cudaMalloc, no
+ * cudaFree, no library routine that allocates.
+ *
+ * pool_dev, pool_bytes: the pool, device memory of `device`; pool_bytes is a
+ *   positive multiple of page_bytes, a power of two in [256 B, 1 GiB].
+ * pages, n_pages: the object's page list in byte order (a host array of
+ *   page indices into the pool, e.g. from t2i_ctl_object), read during the
+ *   call. n_pages = ceil(nbytes / page_bytes), at most 507,520: 64 launches
+ *   of 7,930 pages, one scratch counter each. Larger objects are INVALID.
+ * nbytes: the object's size. dst_dev, dst_bytes: the destination, device
+ *   memory of `device` that does not overlap the pool. cast = 1 writes bf16
+ *   (nbytes % 4 == 0, even dst_dev, dst_bytes >= nbytes / 2); cast = 0
+ *   copies (dst_bytes >= nbytes).
+ * Errors: INVALID (arguments, a page outside the pool, sizes beyond the
+ *   maximum; nothing is enqueued), CUDA (set-up or a launch failed).
+ *   t2i_last_error(NULL) describes them.                                    */
+t2i_status t2i_gather_noalloc(const void* pool_dev, uint64_t pool_bytes, uint64_t page_bytes, const uint32_t* pages,
+                              uint32_t n_pages, uint64_t nbytes, void* dst_dev, uint64_t dst_bytes, uint32_t cast,
+                              int device, void* cuda_stream);
+
+/* =========================================================================
  * First-layer prefix caching (§5.1). A model of L layers keeps its first L_e
  * layers in the store and streams the rest from host memory while inference
  * runs; T_load / T_comp are one layer's load / inference time. Pure host

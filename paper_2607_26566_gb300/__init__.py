@@ -6,5 +6,5 @@ in-tree by :mod:`paper_2607_26566_gb300.build`. This package is its thin
 Python binding; importing :class:`Store` or :class:`Ctl` loads the library and
 fails loudly if it has not been built.
 """
-from .store import (GET_DTYPE, MOVE_DTYPE, PUT_DTYPE, Ctl, Store, T2IError, e2e_latency, get_descs,  # noqa: F401
-                    pipeline_latency, prefix_layers, prefix_layers_pipeline, put_descs)
+from .store import (GET_DTYPE, MOVE_DTYPE, PUT_DTYPE, Ctl, Store, T2IError, e2e_latency, gather_noalloc,  # noqa: F401
+                    get_descs, pipeline_latency, prefix_layers, prefix_layers_pipeline, put_descs)

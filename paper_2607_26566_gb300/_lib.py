@@ -84,6 +84,7 @@ PROTOTYPES = {
     "t2i_ctl_last_evictions": (_S, [_P, _PU64, _U64, _PU64]),
     "t2i_ctl_stats": (_S, [_P, C.POINTER(Stats)]),
     "t2i_ctl_last_error": (C.c_char_p, [_P]),
+    "t2i_gather_noalloc": (_S, [_P, _U64, _U64, _PU32, _U32, _U64, _P, _U64, _U32, C.c_int, _P]),
     "t2i_e2e_latency": (_S, [_U32, _U32, C.c_double, C.c_double, C.POINTER(C.c_double)]),
     "t2i_prefix_layers": (_S, [_U32, C.c_double, C.c_double, _PU32]),
     "t2i_pipeline_latency": (_S, [C.POINTER(C.c_double), C.POINTER(C.c_double), _U32, _U32, C.POINTER(C.c_double)]),

@@ -880,3 +880,208 @@ const char* t2i_last_error(const t2i_store* store) {
 }
 
 }  // extern "C"
+
+// ================================================= gather without allocation
+// t2i_gather_noalloc: the chunked gather of one object's pages for callers
+// that cannot allocate device memory (see include/t2istore.h). Its chunk
+// counters live in a file-scope array that is part of the library's device
+// image, so the call allocates nothing. The paper has no counterpart.
+namespace t2i {
+namespace {
+constexpr uint32_t kNoAllocCounters = 64;  // one per launch of a call: 2 KiB in all
+constexpr uint64_t kNoAllocPagesPerLaunch = (kBlobLarge - sizeof(SegDesc)) / sizeof(uint32_t);
+constexpr int kNoAllocMaxDevices = 64;
+}  // namespace
+}  // namespace t2i
+
+// Every GPU that loads the library holds this array until the process exits.
+static __device__ __align__(256) t2i::WorkCounter t2i_noalloc_scratch[t2i::kNoAllocCounters];
+
+namespace t2i {
+namespace {
+
+// Per-device set-up, done once by the first call on that device: the
+// device address of the scratch array (host code sees only a stand-in for
+// the symbol) and the persistent grid sizes of the gather kernels.
+struct NoAllocDevice {
+    bool ready = false;
+    WorkCounter* scratch = nullptr;
+    int max_ctas[2] = {1, 1};  // [any alignment]
+};
+
+std::mutex g_noalloc_mu;
+NoAllocDevice g_noalloc_dev[kNoAllocMaxDevices];
+
+t2i_status noalloc_setup(int device, NoAllocDevice** out) {
+    std::lock_guard<std::mutex> lock(g_noalloc_mu);
+    NoAllocDevice& d = g_noalloc_dev[device];
+    if (!d.ready) {
+        DeviceGuard g(device);
+        void* ptr = nullptr;
+        cudaError_t e = cudaGetSymbolAddress(&ptr, t2i_noalloc_scratch);
+        if (e != cudaSuccess || !ptr) {
+            set_thread_error(std::string("t2i_gather_noalloc: cannot get the scratch array's device address: ") +
+                             cudaGetErrorString(e));
+            return T2I_ERR_CUDA;
+        }
+        int sms = 0;
+        if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, device) != cudaSuccess || sms <= 0) {
+            set_thread_error("t2i_gather_noalloc: cannot query the device");
+            return T2I_ERR_CUDA;
+        }
+        const void* fns[2] = {reinterpret_cast<const void*>(gather_get_kernel<kBlobLarge, false>),
+                              reinterpret_cast<const void*>(gather_get_kernel<kBlobLarge, true>)};
+        for (int k = 0; k < 2; ++k) {
+            int occ = 0;
+            cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, fns[k], kThreads, 0);
+            d.max_ctas[k] = sms * (occ > 0 ? occ : 1);
+        }
+        d.scratch = static_cast<WorkCounter*>(ptr);
+        d.ready = true;
+    }
+    *out = &d;
+    return T2I_OK;
+}
+
+template <bool GENERAL, int BLOB>
+cudaError_t noalloc_launch(const LaunchParams<BLOB>& p, unsigned grid, cudaStream_t stream) {
+    cudaLaunchConfig_t lc = {};
+    lc.gridDim = dim3(grid);
+    lc.blockDim = dim3(kThreads);
+    lc.stream = stream;
+    void* args[] = {const_cast<LaunchParams<BLOB>*>(&p)};
+    return cudaLaunchKernelExC(&lc, reinterpret_cast<const void*>(gather_get_kernel<BLOB, GENERAL>), args);
+}
+
+// One launch: `np` pages of the object starting at page index `p0`.
+template <bool GENERAL>
+t2i_status noalloc_one(const NoAllocDevice& d, uint32_t k, const void* pool, int shift, const uint32_t* pages,
+                       uint64_t p0, uint64_t np, uint64_t nbytes, unsigned char* dst, bool cast, cudaStream_t stream) {
+    thread_local LaunchParams<kBlobLarge> p;  // host-side parameter staging (no device memory)
+    const uint64_t P = uint64_t(1) << shift;
+    const uint64_t off = p0 * P;
+    const uint64_t seg_bytes = std::min<uint64_t>(nbytes - off, np * P);
+    p.h.pool = reinterpret_cast<uint64_t>(pool);
+    p.h.work = reinterpret_cast<uint64_t>(d.scratch + k);
+    p.h.n_seg = 1;
+    p.h.n_granules = static_cast<uint32_t>((seg_bytes + kGranule - 1) / kGranule);
+    p.h.page_shift = static_cast<uint32_t>(shift);
+    p.h.piece_bytes = static_cast<uint32_t>(std::min<uint64_t>(kPieceBytes, P));
+    p.h.pages_offset = sizeof(SegDesc);
+    p.h.chunk_granules = kChunkGranules;
+    p.h.pad[0] = p.h.pad[1] = 0;
+    SegDesc s;
+    s.user = reinterpret_cast<uint64_t>(dst) + (cast ? off / 2 : off);
+    s.nbytes_flags = seg_bytes | (cast ? kCastFlag : 0);
+    s.start = 0;
+    s.page_begin = 0;
+    std::memcpy(p.blob, &s, sizeof(s));
+    std::memcpy(p.blob + sizeof(SegDesc), pages + p0, np * sizeof(uint32_t));
+    const uint64_t want = (seg_bytes + kMinCtaBytes - 1) / kMinCtaBytes;
+    const unsigned grid =
+        static_cast<unsigned>(std::max<uint64_t>(1, std::min<uint64_t>(want, uint64_t(d.max_ctas[GENERAL ? 1 : 0]))));
+    cudaError_t e = noalloc_launch<GENERAL, kBlobLarge>(p, grid, stream);
+    if (e != cudaSuccess) {
+        set_thread_error(std::string("t2i_gather_noalloc: kernel launch failed: ") + cudaGetErrorString(e));
+        return T2I_ERR_CUDA;
+    }
+    return T2I_OK;
+}
+
+}  // namespace
+}  // namespace t2i
+
+extern "C" t2i_status t2i_gather_noalloc(const void* pool_dev, uint64_t pool_bytes, uint64_t page_bytes,
+                                         const uint32_t* pages, uint32_t n_pages, uint64_t nbytes, void* dst_dev,
+                                         uint64_t dst_bytes, uint32_t cast, int device, void* cuda_stream) {
+    using namespace t2i;
+    NvtxRange nvtx_range(__func__);
+    try {
+        const int shift = log2_exact(page_bytes);
+        if (!pool_dev || shift < 8 || shift > 30 || pool_bytes < page_bytes || pool_bytes % page_bytes != 0 ||
+            cast > 1) {
+            set_thread_error("t2i_gather_noalloc: null pool, page_bytes not a power of two in [256 B, 1 GiB], "
+                             "pool_bytes not a positive multiple of page_bytes, or cast not 0/1");
+            return T2I_ERR_INVALID;
+        }
+        const uint64_t need = nbytes / page_bytes + (nbytes % page_bytes != 0);
+        if (n_pages != need) {
+            set_thread_error("t2i_gather_noalloc: n_pages must be nbytes / page_bytes rounded up");
+            return T2I_ERR_INVALID;
+        }
+        const uint64_t max_pages = uint64_t(kNoAllocCounters) * kNoAllocPagesPerLaunch;
+        if (n_pages > max_pages) {
+            set_thread_error("t2i_gather_noalloc: " + std::to_string(n_pages) + " pages exceed the maximum of " +
+                             std::to_string(max_pages) + " (" + std::to_string(kNoAllocCounters) +
+                             " launches of " + std::to_string(kNoAllocPagesPerLaunch) +
+                             " pages, one scratch counter each)");
+            return T2I_ERR_INVALID;
+        }
+        if (nbytes == 0) return T2I_OK;
+        if (!pages || !dst_dev) {
+            set_thread_error("t2i_gather_noalloc: null page list or destination");
+            return T2I_ERR_INVALID;
+        }
+        if (cast ? (nbytes % 4 != 0 || dst_bytes < nbytes / 2 || (reinterpret_cast<uint64_t>(dst_dev) & 1))
+                 : dst_bytes < nbytes) {
+            set_thread_error("t2i_gather_noalloc: dst_bytes too small, or a cast with nbytes % 4 != 0 or an odd "
+                             "destination address");
+            return T2I_ERR_INVALID;
+        }
+        const uint64_t total_pages = pool_bytes / page_bytes;
+        for (uint32_t i = 0; i < n_pages; ++i)
+            if (pages[i] >= total_pages) {
+                set_thread_error("t2i_gather_noalloc: a page index is outside the pool");
+                return T2I_ERR_INVALID;
+            }
+        int n_dev = 0;
+        if (cudaGetDeviceCount(&n_dev) != cudaSuccess || device < 0 || device >= n_dev ||
+            device >= kNoAllocMaxDevices) {
+            set_thread_error("t2i_gather_noalloc: no such CUDA device");
+            return T2I_ERR_INVALID;
+        }
+        // both ranges must lie in device memory of `device`, and not overlap
+        const uint64_t pa = reinterpret_cast<uint64_t>(pool_dev), da = reinterpret_cast<uint64_t>(dst_dev);
+        const uint64_t dn = cast ? nbytes / 2 : nbytes;
+        Range rp, rd;
+        if (!query_range(pool_dev, &rp) || rp.kind != MemKind::Device || rp.device != device ||
+            pa + pool_bytes > rp.end || !query_range(dst_dev, &rd) || rd.kind != MemKind::Device ||
+            rd.device != device || da + dn > rd.end || da + dn < da) {
+            set_thread_error("t2i_gather_noalloc: the pool and the destination must be device memory of `device` "
+                             "covering their sizes");
+            return T2I_ERR_INVALID;
+        }
+        if (da < pa + pool_bytes && pa < da + dn) {
+            set_thread_error("t2i_gather_noalloc: the destination overlaps the pool");
+            return T2I_ERR_INVALID;
+        }
+        NoAllocDevice* d = nullptr;
+        t2i_status st = noalloc_setup(device, &d);
+        if (st != T2I_OK) return st;
+        DeviceGuard g(device);
+        cudaStream_t stream = static_cast<cudaStream_t>(cuda_stream);
+        const uint64_t n_launch = (n_pages + kNoAllocPagesPerLaunch - 1) / kNoAllocPagesPerLaunch;
+        // the counters this call uses start at zero whatever an earlier call left
+        cudaError_t e = cudaMemsetAsync(d->scratch, 0, n_launch * sizeof(WorkCounter), stream);
+        if (e != cudaSuccess) {
+            set_thread_error(std::string("t2i_gather_noalloc: cannot clear the scratch counters: ") +
+                             cudaGetErrorString(e));
+            return T2I_ERR_CUDA;
+        }
+        const bool general = (da & 15u) != 0;
+        unsigned char* dst = static_cast<unsigned char*>(dst_dev);
+        for (uint64_t k = 0; k < n_launch; ++k) {
+            const uint64_t p0 = k * kNoAllocPagesPerLaunch;
+            const uint64_t np = std::min<uint64_t>(kNoAllocPagesPerLaunch, n_pages - p0);
+            st = general ? noalloc_one<true>(*d, uint32_t(k), pool_dev, shift, pages, p0, np, nbytes, dst, cast != 0,
+                                             stream)
+                         : noalloc_one<false>(*d, uint32_t(k), pool_dev, shift, pages, p0, np, nbytes, dst,
+                                              cast != 0, stream);
+            if (st != T2I_OK) return st;
+        }
+        return T2I_OK;
+    } catch (const std::exception& ex) {
+        set_thread_error(std::string("t2i_gather_noalloc: host error: ") + ex.what());
+        return T2I_ERR_INVALID;
+    }
+}

@@ -325,6 +325,23 @@ class Store:
 
 
 # ---------------------------------------------------------------- prefix caching (§5.1)
+def gather_noalloc(pool, page_bytes: int, pages, nbytes: int, dst, dst_bytes: int | None = None, cast: int = 0,
+                   stream=None, device: int | None = None, pool_bytes: int | None = None) -> int:
+    """t2i_gather_noalloc: one object's pages (``pages``, indices into
+    ``pool``) gathered into ``dst`` with no store and no allocation, for
+    callers that cannot allocate device memory. Returns the status; every
+    call shares the library's static scratch counters, so calls that overlap
+    on the GPU race."""
+    lib = L.load()
+    pg = np.ascontiguousarray(pages, dtype=np.uint32)
+    if device is None:
+        device = int(pool.device.index) if hasattr(pool, "device") else 0
+    return lib.t2i_gather_noalloc(_ptr(pool), int(pool_bytes if pool_bytes is not None else _nbytes(pool)),
+                                  int(page_bytes), pg.ctypes.data_as(C.POINTER(C.c_uint32)), len(pg), int(nbytes),
+                                  _ptr(dst), int(dst_bytes if dst_bytes is not None else _nbytes(dst)), int(cast),
+                                  int(device), _stream(stream))
+
+
 def _dbl(x):
     a = np.ascontiguousarray(x, np.float64)
     return a, a.ctypes.data_as(C.POINTER(C.c_double))
