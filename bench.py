@@ -375,7 +375,10 @@ def time_handoff(hw: Handoff, steps: int, warmup: int, dist_ctx, per_kernel: boo
         # a phase holds hw.requests launches of its kernel, n_streams at a time
         put_ms = statistics.mean(e[0].elapsed_time(e[1]) for e in evs)
         get_ms = statistics.mean(e[1].elapsed_time(e[2]) for e in evs)
+        steps_ms = sorted(e[0].elapsed_time(e[2]) for e in evs)
         kern = {"put_phase_ms": put_ms, "get_phase_ms": get_ms,
+                "step_ms": {"median": round(statistics.median(steps_ms), 4), "best": round(steps_ms[0], 4),
+                            "worst": round(steps_ms[-1], 4), "n": len(steps_ms)},
                 "put_phase_bytes": hw.put_bytes, "get_phase_bytes": hw.get_bytes,
                 "launches_per_phase": hw.requests, "streams": n_streams}
     return ms, launches, kern, (clk.summary() if clk else None)
@@ -1560,6 +1563,7 @@ def main():
                        "bytes_per_step": hw_bytes(B, args.requests), "l2": "inputs > L2 (no flush)",
                        "parallelism": f"replicas x{dist_ctx.world}"},
             "hbm_frac": round(value / dist_ctx.world / peak, 4), "hbm_frac_nominal_8tbs": round(value / dist_ctx.world / 8000.0, 4),
+            "step_ms": kern["step_ms"],
             "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e, "gpu_launches": int(launches),
             "clocks": clocks, "sweep": sweep or None, "extras": extras or None, "rows": rows or None,
         }
