@@ -785,6 +785,33 @@ def time_adapters(device, n_calls: int = 10_000, check_every: int = 500):
     torch.cuda.synchronize(device)
     t_hit = time.perf_counter() - t_hit
     hits_ms = h0.elapsed_time(h1)
+    # the same hit calls with call k on stream k % 4, each stream with its own
+    # destination buffer (four consumers): the gets only read shared pages
+    streams = [stream] + [torch.cuda.Stream(device) for _ in range(3)]
+    bufs = [ad.dst] + [torch.empty_like(ad.dst) for _ in range(3)]
+    desc4 = []
+    for k, d in enumerate(ok_desc):
+        d4 = d.copy()
+        d4["dst"] += np.uint64(bufs[k % 4].data_ptr() - ad.dst.data_ptr())
+        desc4.append(d4)
+    ptr4 = [d.ctypes.data_as(C.POINTER(L.GetDesc)) for d in desc4]
+    ss = [C.c_void_p(x.cuda_stream) for x in streams]
+    h0.record(stream)
+    for x in streams[1:]:
+        x.wait_event(h0)
+    n4 = 0
+    for k, (d, pt) in enumerate(zip(desc4, ptr4)):
+        if lib.t2i_get_batch(h, pt, len(d), None, ss[k % 4]):
+            break
+        n4 += 1
+    for x in streams[1:]:
+        ev = torch.cuda.Event()
+        ev.record(x)
+        stream.wait_event(ev)
+    h1.record(stream)
+    torch.cuda.synchronize(device)
+    hits4_ms = h0.elapsed_time(h1)
+    hit4_bytes = sum(sizes[:n4])
     out = {"workload": "adapters: 512 LoRA sets (ranks 8-64), 16 GiB pool, 256 KiB pages, Zipf(1.1), 256-object gets",
            "calls": n_calls, "ms": round(ms, 2), "calls_per_s": round(n_calls / (ms * 1e-3), 1),
            "wall_calls_per_s": round(n_calls / wall, 1),
@@ -796,6 +823,8 @@ def time_adapters(device, n_calls: int = 10_000, check_every: int = 500):
            "hit_calls": hit_calls, "hit_gbs": round(2 * hit_bytes / (hits_ms * 1e-3) / 1e9, 1),
            "hit_calls_per_s": round(hit_calls / (hits_ms * 1e-3), 1),
            "hit_host_calls_per_s": round(hit_calls / t_hit, 1),
+           "hit_streams4_gbs": round(2 * hit4_bytes / (hits4_ms * 1e-3) / 1e9, 1),
+           "hit_streams4_calls_per_s": round(n4 / (hits4_ms * 1e-3), 1),
            "checked_windows_bad": bad}
     ad.close()
     del ad
@@ -1188,6 +1217,32 @@ def time_pull(device, B: int = 8, requests: int = 64, reps: int = 3):
     e1.record(stream)
     torch.cuda.synchronize(device)
     ms = e0.elapsed_time(e1) / reps
+
+    # the same pulls with request r on stream r % 4 (independent requests overlap)
+    streams = [stream] + [torch.cuda.Stream(device) for _ in range(3)]
+    ss = [C.c_void_p(x.cuda_stream) for x in streams]
+
+    def once4():
+        for r in range(requests):
+            st = lib.t2i_pull(cons._h, hw.store._h, src_p[r], n, 0, dst_p[r], None, ss[r % 4])
+            if st:
+                raise RuntimeError("pull: " + cons.last_error())
+        cons.check(lib.t2i_free(cons._h, new_all, len(new)))
+
+    once4()
+    torch.cuda.synchronize(device)
+    e0.record(stream)
+    for x in streams[1:]:
+        x.wait_event(e0)
+    for _ in range(reps):
+        once4()
+    for x in streams[1:]:
+        ev = torch.cuda.Event()
+        ev.record(x)
+        stream.wait_event(ev)
+    e1.record(stream)
+    torch.cuda.synchronize(device)
+    ms4 = e0.elapsed_time(e1) / reps
     # the consumer's bytes equal the producer's (a sample request)
     from paper_2607_26566_gb300 import get_descs
     st, out, _ = cons.pull(hw.store, hw.ids[:n])
@@ -1197,7 +1252,8 @@ def time_pull(device, B: int = 8, requests: int = 64, reps: int = 3):
     torch.cuda.synchronize(device)
     ok = all(torch.equal(t.reshape(-1).view(torch.uint8), d) for t, d in zip(hw.inputs[0], dst))
     res = {"workload": f"pull: {requests} handoff requests (B={B}) from a producer store into a consumer store",
-           "ms": round(ms, 3), "gbs": round(2 * payload / (ms * 1e-3) / 1e9, 1), "bit_exact": bool(ok)}
+           "ms": round(ms, 3), "gbs": round(2 * payload / (ms * 1e-3) / 1e9, 1), "bit_exact": bool(ok),
+           "streams4_ms": round(ms4, 3), "streams4_gbs": round(2 * payload / (ms4 * 1e-3) / 1e9, 1)}
     cons.close()
     hw.store.close()
     del hw, cons, cons_pool
