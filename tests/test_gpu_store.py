@@ -649,3 +649,47 @@ def test_pull_waits_for_a_late_producer():
     assert cons.get_batch(get_descs([int(iy)], [out]), stream=s2)[0] == 0
     torch.cuda.synchronize()
     assert torch.equal(out, x)
+
+
+def test_chunked_launches_on_eight_streams_at_once():
+    """Large gets (>= 1 MiB per CTA: chunks from the work counters) on eight
+    streams at once, each stream with its own counter; every byte checked,
+    twice in a row (each launch leaves its counter at zero)."""
+    P = 2 << 20
+    n = 600 << 20                                    # 300 pages, 1.3 MiB per CTA of the get grid
+    st = make_store(8 * (n // P) * P + 8 * P, P)
+    streams = [torch.cuda.Stream() for _ in range(8)]
+    xs = [torch.randint(0, 256, (n,), dtype=torch.uint8, device=DEV) for _ in range(8)]
+    s, ids = st.put_batch(put_descs(xs))
+    assert s == 0
+    torch.cuda.synchronize()
+    for _ in range(2):
+        outs = [torch.zeros_like(x) for x in xs]
+        torch.cuda.synchronize()
+        for k in range(8):
+            assert st.get_batch(get_descs([int(ids[k])], [outs[k]]), stream=streams[k])[0] == 0
+        torch.cuda.synchronize()
+        for x, o in zip(xs, outs):
+            assert torch.equal(x, o)
+
+
+def test_streams_beyond_the_counter_slots_split_statically():
+    """A store has work counters for its first 64 streams; later streams use
+    equal static shares. A large get on the 70th stream is still exact."""
+    P = 2 << 20
+    n = 600 << 20
+    st = make_store(n + 8 * P, P)
+    x = torch.randint(0, 256, (n,), dtype=torch.uint8, device=DEV)
+    s, (i,) = st.put_batch(put_descs([x]))
+    assert s == 0
+    streams = [torch.cuda.Stream() for _ in range(70)]
+    small = torch.zeros(64, dtype=torch.uint8, device=DEV)
+    tiny = torch.randint(0, 256, (64,), dtype=torch.uint8, device=DEV)
+    torch.cuda.synchronize()
+    s, (j,) = st.put_batch(put_descs([tiny]))
+    for sm in streams:                                # register 70 streams with the store
+        assert st.get_batch(get_descs([int(j)], [small]), stream=sm)[0] == 0
+    out = torch.zeros_like(x)
+    assert st.get_batch(get_descs([int(i)], [out]), stream=streams[-1])[0] == 0
+    torch.cuda.synchronize()
+    assert torch.equal(out, x) and torch.equal(small, tiny)
