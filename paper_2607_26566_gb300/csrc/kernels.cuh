@@ -5,23 +5,29 @@
 // no host->device descriptor copy.
 //
 // Work split: the segments of a launch are laid end to end in a "launch byte
-// space" (each starting on a 32-byte granule). In a large launch (>= 1 MiB
-// per resident CTA) CTAs take 32 KiB chunks of it one at a time from a
-// counter in device memory (the store's work counter for the launch's
-// stream), so CTAs on SMs that get more bandwidth take more chunks and all
-// CTAs finish within about one chunk of each other: with equal static shares
-// the last CTAs of a large launch finished ~1.6x later than the first on
-// GB300. Smaller launches (work == 0) give each CTA an equal contiguous
-// share. A CTA walks its part in pieces of at most U = 32 KiB that lie in
-// one page of one segment, mapping each piece to its page through the
-// segment's page list.
+// space" (each starting on a 32-byte granule). SMs do not all get the same
+// share of HBM bandwidth: with one equal static share per resident CTA, the
+// last CTAs of a large launch finished ~1.6x later than the first on GB300.
+// So a launch balances its work one of two ways:
+//   - a very large launch (>= 1 MiB per resident CTA) runs a persistent grid
+//     whose CTAs take 32 KiB chunks one at a time from a counter in device
+//     memory (the store's work counter for the launch's stream);
+//   - any other launch (work == 0) runs one CTA per 64 KiB (at least the
+//     resident CTAs, each with >= 16 KiB), each with an equal contiguous
+//     share, and the hardware block scheduler hands CTAs to whichever SMs
+//     free up first.
+// Both leave all CTAs finishing within a chunk or a share of each other. A
+// CTA walks its part in pieces of at most U = 32 KiB that lie in one page of
+// one segment, mapping each piece to its page through the segment's page
+// list.
 //
 // HBM-bound by construction (2 bytes of traffic per payload byte, 1.5 for the
 // cast): fully coalesced 16-byte accesses, enough bytes in flight per SM (8
 // independent 16-byte loads per thread before the first store, 3-4 resident
-// CTAs of 256 threads per SM: 96-128 KiB in flight), a persistent grid sized
-// from the SM count and the occupancy, and programmatic dependent launch so
-// that the next launch's set-up overlaps the end of this one. The launch shape
+// CTAs of 256 threads per SM: 96-128 KiB in flight), grids sized from the SM
+// count, the occupancy and the launch's bytes (see the work split above), and
+// programmatic dependent launch so that the next launch's set-up overlaps the
+// end of this one. The launch shape
 // and cache policy were chosen by a sweep on GB300 (default caching beat
 // streaming hints by ~1.5%; 8 vectors per thread beat 2 and 4).
 #pragma once
@@ -54,6 +60,13 @@ constexpr int kMinBlocksGeneral = 2;  // same, kernels that handle any alignment
 constexpr uint32_t kPieceBytes = kThreads * kVecPerThread * 16;  // U = 32 KiB: one round of the copy loop
 constexpr uint32_t kGranule = 32;  // segment starts and CTA shares fall on 32-byte boundaries
 constexpr uint64_t kMinCtaBytes = 16 * 1024;  // smallest share worth a CTA
+#ifndef T2I_TUNE_STATIC_CTA_BYTES
+#define T2I_TUNE_STATIC_CTA_BYTES (64ull << 10)
+#endif
+// share of a CTA in a large launch without chunks (a sweep: 32, 48, 64, 96,
+// 128, 256 and 512 KiB; 64 KiB was best or within noise of the best on
+// every workload)
+constexpr uint64_t kStaticCtaBytes = T2I_TUNE_STATIC_CTA_BYTES;
 
 // One object segment of a launch. For a put/move the user address is the
 // source; for a get it is the destination. Bit 63 of nbytes_flags asks for

@@ -2,8 +2,8 @@
 // the Store class). A batch's segments are split into 16-byte-aligned and
 // other ones, packed into as few launches as their descriptors allow (each
 // launch carries up to ~31 KiB of descriptors and page numbers in its
-// parameters), and launched as persistent grids with programmatic dependent
-// launch. Together with kernels.cuh this decides what a launch does, so
+// parameters), and launched with programmatic dependent launch: chunked
+// persistent grids for very large launches, else one CTA per 64 KiB. Together with kernels.cuh this decides what a launch does, so
 // profiles are keyed to a hash of both files. Included by store.cu inside
 // namespace t2i.
 #pragma once
@@ -25,11 +25,18 @@ t2i_status Store::launch_one(const std::vector<SegDesc>& sd, const std::vector<u
     p->h.pages_offset = static_cast<uint32_t>(sd.size() * sizeof(SegDesc));
     std::memcpy(p->blob, sd.data(), sd.size() * sizeof(SegDesc));
     std::memcpy(p->blob + p->h.pages_offset, pages.data(), pages.size() * sizeof(uint32_t));
-    // every CTA gets at least kMinCtaBytes of the launch (small batches use a
-    // smaller grid); at most the resident CTAs of the whole device
-    const uint64_t want = (uint64_t(n_granules) * kGranule + kMinCtaBytes - 1) / kMinCtaBytes;
-    const unsigned grid = static_cast<unsigned>(
-        std::max<uint64_t>(1, std::min<uint64_t>(want, uint64_t(max_ctas_[int(M)][GENERAL ? 1 : 0]))));
+    // Grid. A chunked launch is persistent: the resident CTAs of the device.
+    // Otherwise CTAs take equal static shares of 16-64 KiB: the resident CTAs
+    // while that gives each at least kMinCtaBytes, and one CTA per
+    // kStaticCtaBytes beyond, so that the hardware hands the CTAs of a larger
+    // launch to whichever SMs free up first.
+    const uint64_t bytes = uint64_t(n_granules) * kGranule;
+    const uint64_t resident = uint64_t(max_ctas_[int(M)][GENERAL ? 1 : 0]);
+    const uint64_t want = (bytes + kMinCtaBytes - 1) / kMinCtaBytes;
+    uint64_t g = std::max<uint64_t>(1, std::min<uint64_t>(want, resident));
+    if (p->h.work == 0) g = std::max<uint64_t>(g, std::min<uint64_t>((bytes + kStaticCtaBytes - 1) / kStaticCtaBytes,
+                                                                     0x7FFFFFFFull));
+    const unsigned grid = static_cast<unsigned>(g);
     void* args[] = {p};
     const void* fn = M == Mode::Put   ? reinterpret_cast<const void*>(scatter_put_kernel<BLOB, GENERAL>)
                      : M == Mode::Get ? reinterpret_cast<const void*>(gather_get_kernel<BLOB, GENERAL>)

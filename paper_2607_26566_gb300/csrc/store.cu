@@ -130,7 +130,7 @@ class Store {
             *err = "cannot query the device";
             return T2I_ERR_CUDA;
         }
-        // persistent grids: resident CTAs per SM x SMs, per kernel
+        // resident CTAs on the device (SMs x CTAs per SM), per kernel
         const void* fns[3][2] = {
             {reinterpret_cast<const void*>(scatter_put_kernel<kBlobLarge, false>),
              reinterpret_cast<const void*>(scatter_put_kernel<kBlobLarge, true>)},
@@ -902,7 +902,7 @@ namespace {
 
 // Per-device set-up, done once by the first call on that device: the
 // device address of the scratch array (host code sees only a stand-in for
-// the symbol) and the persistent grid sizes of the gather kernels.
+// the symbol) and the resident CTAs of the gather kernels (its grid size).
 struct NoAllocDevice {
     bool ready = false;
     WorkCounter* scratch = nullptr;
