@@ -62,6 +62,8 @@ def parse():
     p.add_argument("--rows", default="tiny,weights,adapters,compaction,prefix,views,pull",
                    help="other hot-path rows timed in the same run (comma list, or 'none')")
     p.add_argument("--adapter-calls", type=int, default=10_000)
+    p.add_argument("--adapter-sets", type=int, default=None, help="fewer LoRA sets (profiling small cases)")
+    p.add_argument("--adapter-pool-gib", type=float, default=None, help="smaller adapter pool (profiling small cases)")
     p.add_argument("--rows-only", action="store_true", help="skip the handoff headline (profiling a row)")
     p.add_argument("--weight-blocks", type=int, default=None,
                    help="restore only the first N blocks into a pool sized for them (profiling small cases)")
@@ -732,10 +734,11 @@ class Adapters:
         self.store.close()
 
 
-def time_adapters(device, n_calls: int = 10_000, check_every: int = 500):
+def time_adapters(device, n_calls: int = 10_000, check_every: int = 500, n_sets: int | None = None,
+                  pool_bytes: int | None = None):
     import torch
 
-    ad = Adapters(device, n_calls=n_calls)
+    ad = Adapters(device, n_calls=n_calls, n_sets=n_sets or W.ADAPTERS["n_sets"], pool_bytes=pool_bytes)
     ad.load_events = []
     stream = torch.cuda.current_stream(device)
     torch.cuda.synchronize(device)
@@ -812,7 +815,10 @@ def time_adapters(device, n_calls: int = 10_000, check_every: int = 500):
     torch.cuda.synchronize(device)
     hits4_ms = h0.elapsed_time(h1)
     hit4_bytes = sum(sizes[:n4])
-    out = {"workload": "adapters: 512 LoRA sets (ranks 8-64), 16 GiB pool, 256 KiB pages, Zipf(1.1), 256-object gets",
+    small = n_sets is not None or pool_bytes is not None
+    out = {"workload": ("adapters: 512 LoRA sets (ranks 8-64), 16 GiB pool, 256 KiB pages, Zipf(1.1), 256-object gets"
+                        if not small else f"adapters (small case): {len(ad.ranks)} sets, "
+                                          f"{ad.pool.numel() / 2**30:.1f} GiB pool"),
            "calls": n_calls, "ms": round(ms, 2), "calls_per_s": round(n_calls / (ms * 1e-3), 1),
            "wall_calls_per_s": round(n_calls / wall, 1),
            "window_misses": ad.window_misses, "reloads": ad.loads, "reloaded_objects": ad.load_objects,
@@ -1446,7 +1452,9 @@ def run_rows(args, device, peak):
     if "weights" in wanted:
         rows["weights"] = time_weights(device, n_blocks=args.weight_blocks)
     if "adapters" in wanted:
-        rows["adapters"] = time_adapters(device, n_calls=args.adapter_calls)
+        rows["adapters"] = time_adapters(device, n_calls=args.adapter_calls, n_sets=args.adapter_sets,
+                                         pool_bytes=int(args.adapter_pool_gib * (1 << 30)) if args.adapter_pool_gib
+                                         else None)
     if "compaction" in wanted:
         rows["compaction"] = time_compaction(device, pool_gib=args.compaction_gib)
     if "prefix" in wanted:

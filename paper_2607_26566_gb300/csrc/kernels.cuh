@@ -67,6 +67,10 @@ constexpr uint64_t kMinCtaBytes = 16 * 1024;  // smallest share worth a CTA
 // 128, 256 and 512 KiB; 64 KiB was best or within noise of the best on
 // every workload)
 constexpr uint64_t kStaticCtaBytes = T2I_TUNE_STATIC_CTA_BYTES;
+#ifndef T2I_TUNE_GET_COPY_KERNEL
+#define T2I_TUNE_GET_COPY_KERNEL 1
+#endif
+constexpr bool kGetCopyKernel = T2I_TUNE_GET_COPY_KERNEL != 0;  // gets without casts run gather_copy_kernel
 
 // One object segment of a launch. For a put/move the user address is the
 // source; for a get it is the destination. Bit 63 of nbytes_flags asks for
@@ -127,7 +131,8 @@ constexpr int kBlobSmall = 1024;
 constexpr int kBlobMid = 8192;
 constexpr int kBlobLarge = 31 * 1024;  // header + blob stays below the 32,764-byte parameter limit
 
-enum class Mode { Put, Get, Move };
+// GetCopy: a get whose launch has no cast segment (a leaner kernel).
+enum class Mode { Put, Get, Move, GetCopy };
 
 #ifdef __CUDACC__
 
@@ -432,8 +437,8 @@ __device__ __forceinline__ void run_range(const LaunchParams<BLOB>& p, uint64_t 
         const uint32_t len = (uint32_t)umin64(umin64(end - pos, nbytes - off), umin64(piece, pmask + 1 - in_page));
         unsigned char* paddr = page_base + in_page;
         unsigned char* uaddr = reinterpret_cast<unsigned char*>(s.user);
-        if (M == Mode::Get) {
-            if (s.nbytes_flags & kCastFlag) {
+        if (M == Mode::Get || M == Mode::GetCopy) {
+            if (M == Mode::Get && (s.nbytes_flags & kCastFlag)) {
                 if (!GENERAL || (reinterpret_cast<uintptr_t>(uaddr) & 15u) == 0)
                     cta_cast_aligned<kV>(uaddr + (off >> 1), paddr, len);
                 else
@@ -465,6 +470,13 @@ __global__ void __launch_bounds__(kThreads, GENERAL ? kMinBlocksGeneral : kMinBl
     gather_get_kernel(const __grid_constant__ LaunchParams<BLOB> p) {
     pdl_wait_then_release();
     run_share<Mode::Get, GENERAL, BLOB>(p);
+}
+// A get launch without casts: the copy path alone fits the register budget
+// of kMinBlocks resident CTAs, like the put.
+template <int BLOB>
+__global__ void __launch_bounds__(kThreads, kMinBlocks) gather_copy_kernel(const __grid_constant__ LaunchParams<BLOB> p) {
+    pdl_wait_then_release();
+    run_share<Mode::GetCopy, false, BLOB>(p);
 }
 template <int BLOB>
 __global__ void __launch_bounds__(kThreads, kMinBlocks) compact_move_kernel(const __grid_constant__ LaunchParams<BLOB> p) {

@@ -131,14 +131,16 @@ class Store {
             return T2I_ERR_CUDA;
         }
         // resident CTAs on the device (SMs x CTAs per SM), per kernel
-        const void* fns[3][2] = {
+        const void* fns[4][2] = {
             {reinterpret_cast<const void*>(scatter_put_kernel<kBlobLarge, false>),
              reinterpret_cast<const void*>(scatter_put_kernel<kBlobLarge, true>)},
             {reinterpret_cast<const void*>(gather_get_kernel<kBlobLarge, false>),
              reinterpret_cast<const void*>(gather_get_kernel<kBlobLarge, true>)},
             {reinterpret_cast<const void*>(compact_move_kernel<kBlobLarge>),
-             reinterpret_cast<const void*>(compact_move_kernel<kBlobLarge>)}};
-        for (int m = 0; m < 3; ++m)
+             reinterpret_cast<const void*>(compact_move_kernel<kBlobLarge>)},
+            {reinterpret_cast<const void*>(gather_copy_kernel<kBlobLarge>),
+             reinterpret_cast<const void*>(gather_copy_kernel<kBlobLarge>)}};
+        for (int m = 0; m < 4; ++m)
             for (int g = 0; g < 2; ++g) {
                 int occ = 0;
                 cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, fns[m][g], kThreads, 0);
@@ -231,7 +233,7 @@ class Store {
     Control ctl_;
     t2i_ctl handle_{};
     uint32_t page_shift_ = 0;
-    int max_ctas_[3][2] = {{1, 1}, {1, 1}, {1, 1}};  // [mode][any alignment]: resident CTAs on the device
+    int max_ctas_[4][2] = {{1, 1}, {1, 1}, {1, 1}, {1, 1}};  // [mode][any alignment]: resident CTAs on the device
     uint32_t fail_countdown_ = 0;  // > 0: that many launches from now, report a failure (testing)
     // Work counters, one per stream index: launches on one stream run one
     // after another (each waits for the previous grid before touching its
