@@ -1,6 +1,8 @@
 // Host control core: see control.hpp for the rules it implements.
 #include "control.hpp"
 
+#include <cstdint>
+
 #include <algorithm>
 #include <string>
 
@@ -239,6 +241,8 @@ t2i_status Control::view(uint64_t id, const Object** out) {
 }
 
 void Control::rollback_compact() {
+    // the free pages and the limit change only in finish_compact: the page
+    // tables and the counters are all there is to undo
     for (const Remap& r : last_remap_) {
         page_obj_[r.o->pages[r.idx]] = nullptr;
         r.o->pages[r.idx] = r.old_page;
@@ -246,9 +250,6 @@ void Control::rollback_compact() {
         page_idx_[r.old_page] = r.idx;
     }
     last_remap_.clear();
-    free_.restore(std::move(last_free_));
-    last_free_ = FreePages::Snapshot{};
-    limit_pages_ = last_limit_;
     counters_.pages_moved = last_compact_counters_.pages_moved;
     counters_.bytes_moved = last_compact_counters_.bytes_moved;
 }
@@ -489,6 +490,14 @@ t2i_status Control::compact(uint64_t limit_bytes, std::vector<t2i_move>* moves) 
 
 t2i_status Control::plan_compact(uint64_t limit_bytes, std::vector<t2i_move>* moves) {
     moves->clear();
+    const t2i_status st = begin_compact(limit_bytes);
+    if (st != T2I_OK) return st;
+    moves->reserve(last_remap_.capacity());
+    plan_more(SIZE_MAX, moves);
+    return T2I_OK;
+}
+
+t2i_status Control::begin_compact(uint64_t limit_bytes) {
     if (limit_bytes % P_ != 0 || limit_bytes / P_ > total_pages_) {
         err_ = "compact: the limit must be a multiple of the page size and at most the pool";
         return T2I_ERR_INVALID;
@@ -498,21 +507,26 @@ t2i_status Control::plan_compact(uint64_t limit_bytes, std::vector<t2i_move>* mo
         err_ = "compact: more pages are in use than the limit holds";
         return T2I_ERR_NOSPACE;
     }
-    moves->reserve(live_pages_at_or_above(limit));
     last_remap_.clear();
-    last_remap_.reserve(moves->capacity());
-    last_free_ = free_.snapshot();
-    last_limit_ = limit_pages_;
+    last_remap_.reserve(live_pages_at_or_above(limit));
     last_compact_counters_ = counters_;
+    planned_limit_ = limit;
+    plan_p_ = limit;
+    plan_scan_ = 0;
+    return T2I_OK;
+}
+
+bool Control::plan_more(size_t max, std::vector<t2i_move>* moves) {
     // live pages at or above the limit, ascending (pages at or above the
     // current limit are all free), each to the lowest free page below it
-    uint64_t scan = 0;
+    size_t n = 0;
     uint64_t moved_bytes = 0;
-    for (uint64_t p = limit; p < limit_pages_; ++p) {
+    for (; plan_p_ < limit_pages_ && n < max; ++plan_p_) {
+        const uint64_t p = plan_p_;
         Object* o = page_obj_[p];
         if (!o) continue;
-        while (page_obj_[scan]) ++scan;  // used_pages_ <= limit guarantees a free page
-        const uint32_t dst = static_cast<uint32_t>(scan);
+        while (page_obj_[plan_scan_]) ++plan_scan_;  // used_pages_ <= limit guarantees a free page
+        const uint32_t dst = static_cast<uint32_t>(plan_scan_);
         const uint32_t idx = page_idx_[p];
         const uint64_t valid = std::min<uint64_t>(P_, o->nbytes - uint64_t(idx) * P_);
         o->pages[idx] = dst;
@@ -522,11 +536,14 @@ t2i_status Control::plan_compact(uint64_t limit_bytes, std::vector<t2i_move>* mo
         last_remap_.push_back({o, idx, static_cast<uint32_t>(p)});
         moves->push_back({static_cast<uint32_t>(p), dst, valid});
         moved_bytes += valid;
+        ++n;
     }
-    planned_limit_ = limit;
-    counters_.pages_moved += moves->size();
+    counters_.pages_moved += n;
     counters_.bytes_moved += moved_bytes;
-    return T2I_OK;
+    // more to plan if a live page may remain at or above the limit
+    for (; plan_p_ < limit_pages_; ++plan_p_)
+        if (page_obj_[plan_p_]) return true;
+    return false;
 }
 
 void Control::finish_compact() {

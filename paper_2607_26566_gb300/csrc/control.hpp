@@ -80,18 +80,6 @@ class FreePages {
     // an object's pages back, in page-list order (or, undoing a take, in
     // reverse, which restores a LIFO stack exactly)
     void give(const std::vector<uint32_t>& pages, bool undo = false);
-    // the whole structure, for undoing a compaction
-    struct Snapshot {
-        uint64_t count;
-        std::vector<uint32_t> stack;
-        std::map<uint32_t, uint32_t> runs;
-    };
-    Snapshot snapshot() const { return {count_, stack_, runs_}; }
-    void restore(Snapshot s) {
-        count_ = s.count;
-        stack_ = std::move(s.stack);
-        runs_ = std::move(s.runs);
-    }
     // after a compaction: every page below limit for which used(p) is false
     template <class Used>
     void rebuild(uint64_t limit, Used used) {
@@ -182,14 +170,20 @@ class Control {
     t2i_status free(const t2i_id* ids, uint32_t n);
     // compact: plans, remaps and returns the moves (always filled).
     t2i_status compact(uint64_t limit_bytes, std::vector<t2i_move>* moves);
-    // The same in two halves, so that the free pages can be rebuilt while
-    // the moves run: plan_compact remaps and returns the moves;
-    // finish_compact (after a successful plan, before any other call)
-    // rebuilds the free pages and applies the new limit.
+    // The same in steps, so that moves can run while the rest is planned
+    // and the free pages are rebuilt while the moves run:
+    //   begin_compact validates the limit and starts a plan;
+    //   plan_more remaps up to `max` more live pages and appends their moves
+    //     (true while live pages remain at or above the limit);
+    //   finish_compact (after a complete plan, before any other call)
+    //     rebuilds the free pages and applies the new limit;
+    //   rollback_compact (instead of finish_compact, after a failed launch)
+    //     puts every page list planned since begin_compact back.
+    // plan_compact is begin_compact + plan_more until done.
     t2i_status plan_compact(uint64_t limit_bytes, std::vector<t2i_move>* moves);
+    t2i_status begin_compact(uint64_t limit_bytes);
+    bool plan_more(size_t max, std::vector<t2i_move>* moves);
     void finish_compact();
-    // Undo the last compaction (after a failed launch): page lists, the free
-    // pages and the limit return to their state before it.
     void rollback_compact();
 
     uint64_t live_pages_at_or_above(uint64_t limit) const;
@@ -243,9 +237,9 @@ class Control {
     std::vector<Object*> page_obj_;
     std::vector<uint32_t> page_idx_;
     std::vector<Remap> last_remap_;          // the last compaction, for rollback_compact
-    FreePages::Snapshot last_free_;
-    uint64_t last_limit_ = 0;
     uint64_t planned_limit_ = 0;
+    uint64_t plan_p_ = 0;      // next page at or above the limit to look at
+    uint64_t plan_scan_ = 0;   // lowest page below the limit that may be free
     t2i_stats last_compact_counters_{};
     t2i_stats counters_{};
     std::string err_;

@@ -246,6 +246,10 @@ class Store {
     std::string err_;
     std::vector<const Object*> objs_;
     std::vector<Seg> segs_;
+    std::vector<t2i_move> batch_;  // the moves of one compaction launch
+    // moves per compaction launch: one 24-byte descriptor and one page each
+    static constexpr size_t kMovesPerLaunch = 1024;
+    static_assert(kMovesPerLaunch * (sizeof(SegDesc) + sizeof(uint32_t)) <= size_t(kBlobLarge), "moves per launch");
     std::vector<SegDesc> sd_;
     std::vector<uint32_t> lp_;
     alignas(16) unsigned char param_buf_[sizeof(LaunchParams<kBlobLarge>)];
@@ -634,58 +638,65 @@ t2i_status Store::pull_from(Store& src, const t2i_id* ids, uint32_t n, uint32_t 
 }
 
 t2i_status Store::compact(uint64_t limit_bytes, cudaStream_t stream, uint64_t* moved) {
-    std::vector<t2i_move> moves;
-    t2i_status st = ctl_.plan_compact(limit_bytes, &moves);
-    if (moved) *moved = moves.size();
+    if (moved) *moved = 0;
+    t2i_status st = ctl_.begin_compact(limit_bytes);
     if (st != T2I_OK) {
         err_ = ctl_.error();
         return st;
-    }
-    if (moves.empty()) {
-        ctl_.finish_compact();
-        return T2I_OK;
     }
     DeviceGuard g(device_);
     int si = 0;
     if ((st = stream_slot(stream, &si)) != T2I_OK) {
         ctl_.rollback_compact();
-        if (moved) *moved = 0;
         return st;
     }
-    deps_.begin(si);
-    for (const t2i_move& m : moves) {
-        deps_.reads(m.src_page);
-        deps_.writes(m.dst_page);
-    }
-    cudaError_t we = deps_.wait();
-    if (we != cudaSuccess) {
-        ctl_.rollback_compact();
-        if (moved) *moved = 0;
-        return cuda_fail("compact: cannot order after earlier calls", we);
-    }
-    segs_.clear();
+    // Planned and launched one launch's worth of moves at a time, so that the
+    // first moves run while the rest is planned.
     const uint64_t P = uint64_t(1) << page_shift_;
-    // each move is a one-page segment whose source is the old page
-    for (const t2i_move& m : moves)
-        segs_.push_back({pool_ + uint64_t(m.src_page) * P, m.valid_bytes, &m.dst_page, 1u});
-    st = launch_segments<Mode::Move>(segs_, stream);
-    // marked even after a failure part-way: moves launched before it may
-    // still be reading the old pages and writing the new ones
-    uint32_t q = 0;
-    cudaError_t ee = deps_.end(&q);
-    for (const t2i_move& m : moves) {
-        deps_.mark_read(m.src_page, q);
-        deps_.mark_write(m.dst_page, q);
-    }
-    if (st != T2I_OK) {
-        // the old pages still hold every byte: point the page tables back
-        ctl_.rollback_compact();
-        if (moved) *moved = 0;
-        return st;
+    uint64_t total = 0;
+    cudaError_t event_error = cudaSuccess;
+    bool more = true;
+    while (more) {
+        batch_.clear();
+        more = ctl_.plan_more(kMovesPerLaunch, &batch_);
+        if (batch_.empty()) break;
+        deps_.begin(si);
+        if (deps_.n_streams() > 1) {  // with one stream there is nothing to wait for
+            for (const t2i_move& m : batch_) {
+                deps_.reads(m.src_page);
+                deps_.writes(m.dst_page);
+            }
+        }
+        cudaError_t we = deps_.wait();
+        if (we != cudaSuccess) {
+            ctl_.rollback_compact();
+            return cuda_fail("compact: cannot order after earlier calls", we);
+        }
+        segs_.clear();
+        // each move is a one-page segment whose source is the old page
+        for (const t2i_move& m : batch_)
+            segs_.push_back({pool_ + uint64_t(m.src_page) * P, m.valid_bytes, &m.dst_page, 1u});
+        st = launch_segments<Mode::Move>(segs_, stream);
+        // marked even after a failure: launches before it may still be
+        // reading the old pages and writing the new ones
+        uint32_t q = 0;
+        cudaError_t ee = deps_.end(&q);
+        for (const t2i_move& m : batch_) {
+            deps_.mark_read(m.src_page, q);
+            deps_.mark_write(m.dst_page, q);
+        }
+        if (st != T2I_OK) {
+            // the old pages still hold every byte: point the page tables back
+            ctl_.rollback_compact();
+            return st;
+        }
+        if (ee != cudaSuccess && event_error == cudaSuccess) event_error = ee;
+        total += batch_.size();
     }
     ctl_.finish_compact();  // the free pages are rebuilt while the moves run
-    if (ee != cudaSuccess) st = cuda_fail("compact: cannot record its event", ee);
-    return st;
+    if (moved) *moved = total;
+    if (event_error != cudaSuccess) return cuda_fail("compact: cannot record its event", event_error);
+    return T2I_OK;
 }
 
 }  // namespace t2i
