@@ -141,10 +141,10 @@ class Store {
             {reinterpret_cast<const void*>(gather_copy_kernel<kBlobLarge>),
              reinterpret_cast<const void*>(gather_copy_kernel<kBlobLarge>)}};
         for (int m = 0; m < 4; ++m)
-            for (int g = 0; g < 2; ++g) {
+            for (int a = 0; a < 2; ++a) {
                 int occ = 0;
-                cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, fns[m][g], kThreads, 0);
-                max_ctas_[m][g] = sms * (occ > 0 ? occ : 1);
+                cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, fns[m][a], kThreads, 0);
+                max_ctas_[m][a] = sms * (occ > 0 ? occ : 1);
             }
         // one chunk counter per stream (the first kWorkStreams streams of
         // the store; later ones use equal static shares), zeroed once
