@@ -100,7 +100,9 @@ t2i_status Store::launch_group(const std::vector<Seg>& segs, cudaStream_t stream
         if (sd_.empty()) return T2I_OK;
         const size_t bytes = sd_.size() * sizeof(SegDesc) + lp_.size() * sizeof(uint32_t);
         t2i_status st;
-        if (bytes <= size_t(kBlobSmall))
+        if (bytes <= size_t(kBlobTiny))
+            st = launch_one<M, GENERAL, kBlobTiny>(sd_, lp_, uint32_t(gran), stream);
+        else if (bytes <= size_t(kBlobSmall))
             st = launch_one<M, GENERAL, kBlobSmall>(sd_, lp_, uint32_t(gran), stream);
         else if (bytes <= size_t(kBlobMid))
             st = launch_one<M, GENERAL, kBlobMid>(sd_, lp_, uint32_t(gran), stream);

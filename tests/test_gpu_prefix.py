@@ -27,7 +27,9 @@ def test_layer_streaming_bytes_and_overlap():
     comp = [pp.t_sleep + g for g in pp.t_get]
     le = prefix_layers_pipeline(pp.t_load, comp)
     assert 0 < le < pp.L
-    t_none = pp.request(0)
+    # the best of two requests: the host link is shared with other work on
+    # the machine, and one slow transfer should not decide the comparison
+    t_none = min(pp.request(0), pp.request(0))
     # every block got during the request equals its pinned host bytes
     for b in range(pp.L):
         st, _ = pp.store.get_batch(pp._layer_gd(b), stream=pp.s_comp, per_item=False)
@@ -38,7 +40,7 @@ def test_layer_streaming_bytes_and_overlap():
         for i, off in members:
             n = pp.wr.specs[i].nbytes
             assert torch.equal(pp.work[off:off + n].cpu(), h[off:off + n]), (b, i)
-    t_cached = pp.request(le)
+    t_cached = min(pp.request(le), pp.request(le))
     # loading is hidden: the cached request is faster and close to the model
     assert t_cached < t_none
     model_none = pipeline_latency(pp.t_load, comp, 0)
