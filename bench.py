@@ -1564,6 +1564,22 @@ def main():
             ms_s, _, _, _ = time_handoff(hs, max(3, args.steps // 2), args.warmup, dist_ctx, per_kernel=False,
                                          n_streams=args.streams, nvtx="bench_sweep")
             sweep[f"B{Bs}"] = round(hs.step_bytes * max(3, args.steps // 2) / (ms_s * 1e-3) / 1e9, 1)
+            if Bs == 1:
+                # small requests: the same on one stream, and one call per phase
+                ms_1, _, _, _ = time_handoff(hs, max(3, args.steps // 2), args.warmup, dist_ctx, per_kernel=False,
+                                             nvtx="bench_sweep")
+                sweep["B1_one_stream"] = round(hs.step_bytes * max(3, args.steps // 2) / (ms_1 * 1e-3) / 1e9, 1)
+                stream = torch.cuda.current_stream(device)
+                for _ in range(3):
+                    hs.step_one_call()
+                torch.cuda.synchronize(device)
+                a, z = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                a.record(stream)
+                for _ in range(10):
+                    hs.step_one_call()
+                z.record(stream)
+                torch.cuda.synchronize(device)
+                sweep["B1_one_call_per_phase"] = round(hs.step_bytes * 10 / (a.elapsed_time(z) * 1e-3) / 1e9, 1)
             del hs
             torch.cuda.empty_cache()
 
