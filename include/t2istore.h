@@ -321,8 +321,9 @@ t2i_status t2i_inject_launch_failure(t2i_store* store, uint32_t countdown);
  *   positive multiple of page_bytes, a power of two in [256 B, 1 GiB].
  * pages, n_pages: the object's page list in byte order (a host array of
  *   page indices into the pool, e.g. from t2i_ctl_object), read during the
- *   call. n_pages = ceil(nbytes / page_bytes), at most 507,520: 64 launches
- *   of 7,930 pages, one scratch counter each. Larger objects are INVALID.
+ *   call. n_pages = ceil(nbytes / page_bytes), at most 64 launches of
+ *   min(7,930, 64 GiB / page_bytes) pages, one scratch counter each: 507,520
+ *   pages for pages up to 8 MiB. Larger objects are INVALID.
  * nbytes: the object's size. dst_dev, dst_bytes: the destination, device
  *   memory of `device` that does not overlap the pool. cast = 1 writes bf16
  *   (nbytes % 4 == 0, even dst_dev, dst_bytes >= nbytes / 2); cast = 0

@@ -132,6 +132,9 @@ struct LaunchParams {
 // B=1 handoff request, 124 bytes of descriptors, ran the 4-stream B=1 step
 // 4% faster than the 1 KiB tier).
 constexpr int kBlobTiny = 256;
+// Largest segment (bytes) of one launch: 2^31 granules, so that granule
+// offsets of a launch (32-bit) never wrap.
+constexpr uint64_t kMaxSegBytes = uint64_t(1) << 36;
 constexpr int kBlobSmall = 1024;
 constexpr int kBlobMid = 8192;
 constexpr int kBlobLarge = 31 * 1024;  // header + blob stays below the 32,764-byte parameter limit

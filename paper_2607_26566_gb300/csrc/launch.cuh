@@ -114,7 +114,10 @@ t2i_status Store::launch_group(const std::vector<Seg>& segs, cudaStream_t stream
         return st;
     };
     const uint64_t P = uint64_t(1) << page_shift_;
-    const uint64_t max_pages_per_seg = (kBlobLarge - sizeof(SegDesc)) / sizeof(uint32_t);
+    // a segment's page list fits one launch, and its bytes fit the 32-bit
+    // granule offsets of the launch byte space (64 GiB per segment)
+    const uint64_t max_pages_per_seg = std::min<uint64_t>((kBlobLarge - sizeof(SegDesc)) / sizeof(uint32_t),
+                                                          std::max<uint64_t>(1, kMaxSegBytes / P));
     for (const Seg& s : segs) {
         const uint64_t nbytes = s.nbytes_flags & ~kCastFlag;
         const uint64_t flags = s.nbytes_flags & kCastFlag;

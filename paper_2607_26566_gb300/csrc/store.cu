@@ -902,7 +902,12 @@ const char* t2i_last_error(const t2i_store* store) {
 namespace t2i {
 namespace {
 constexpr uint32_t kNoAllocCounters = 64;  // one per launch of a call: 2 KiB in all
-constexpr uint64_t kNoAllocPagesPerLaunch = (kBlobLarge - sizeof(SegDesc)) / sizeof(uint32_t);
+constexpr uint64_t kNoAllocMaxPagesPerLaunch = (kBlobLarge - sizeof(SegDesc)) / sizeof(uint32_t);
+// pages per launch: the page list fits the parameters and the bytes fit
+// 32-bit granule offsets
+uint64_t noalloc_pages_per_launch(uint64_t page_bytes) {
+    return std::min<uint64_t>(kNoAllocMaxPagesPerLaunch, std::max<uint64_t>(1, kMaxSegBytes / page_bytes));
+}
 constexpr int kNoAllocMaxDevices = 64;
 }  // namespace
 }  // namespace t2i
@@ -1022,12 +1027,12 @@ extern "C" t2i_status t2i_gather_noalloc(const void* pool_dev, uint64_t pool_byt
             set_thread_error("t2i_gather_noalloc: n_pages must be nbytes / page_bytes rounded up");
             return T2I_ERR_INVALID;
         }
-        const uint64_t max_pages = uint64_t(kNoAllocCounters) * kNoAllocPagesPerLaunch;
+        const uint64_t per_launch = noalloc_pages_per_launch(page_bytes);
+        const uint64_t max_pages = uint64_t(kNoAllocCounters) * per_launch;
         if (n_pages > max_pages) {
             set_thread_error("t2i_gather_noalloc: " + std::to_string(n_pages) + " pages exceed the maximum of " +
                              std::to_string(max_pages) + " (" + std::to_string(kNoAllocCounters) +
-                             " launches of " + std::to_string(kNoAllocPagesPerLaunch) +
-                             " pages, one scratch counter each)");
+                             " launches of " + std::to_string(per_launch) + " pages, one scratch counter each)");
             return T2I_ERR_INVALID;
         }
         if (nbytes == 0) return T2I_OK;
@@ -1073,7 +1078,7 @@ extern "C" t2i_status t2i_gather_noalloc(const void* pool_dev, uint64_t pool_byt
         if (st != T2I_OK) return st;
         DeviceGuard g(device);
         cudaStream_t stream = static_cast<cudaStream_t>(cuda_stream);
-        const uint64_t n_launch = (n_pages + kNoAllocPagesPerLaunch - 1) / kNoAllocPagesPerLaunch;
+        const uint64_t n_launch = (n_pages + per_launch - 1) / per_launch;
         // the counters this call uses start at zero whatever an earlier call left
         cudaError_t e = cudaMemsetAsync(d->scratch, 0, n_launch * sizeof(WorkCounter), stream);
         if (e != cudaSuccess) {
@@ -1084,8 +1089,8 @@ extern "C" t2i_status t2i_gather_noalloc(const void* pool_dev, uint64_t pool_byt
         const bool general = (da & 15u) != 0;
         unsigned char* dst = static_cast<unsigned char*>(dst_dev);
         for (uint64_t k = 0; k < n_launch; ++k) {
-            const uint64_t p0 = k * kNoAllocPagesPerLaunch;
-            const uint64_t np = std::min<uint64_t>(kNoAllocPagesPerLaunch, n_pages - p0);
+            const uint64_t p0 = k * per_launch;
+            const uint64_t np = std::min<uint64_t>(per_launch, n_pages - p0);
             st = general ? noalloc_one<true>(*d, uint32_t(k), pool_dev, shift, pages, p0, np, nbytes, dst, cast != 0,
                                              stream)
                          : noalloc_one<false>(*d, uint32_t(k), pool_dev, shift, pages, p0, np, nbytes, dst,

@@ -113,3 +113,30 @@ def test_unaligned_cast_and_copy_kernels():
         got = bf.cpu().numpy()[e:e + f.nbytes // 2].view(np.uint16)
         assert np.array_equal(got, f32_bits_to_bf16_bits(f.view(np.uint32)))
         assert st.free([int(i)]) == 0
+
+
+def test_object_larger_than_64_gib():
+    """An object of 65 GiB + a ragged tail in 1 GiB pages: its launch byte
+    space is split into segments of at most 64 GiB, so 32-bit granule
+    offsets never wrap. Every GiB of the get is compared with the put."""
+    G = 1 << 30
+    if torch.cuda.get_device_properties(0).total_memory < 180 * G:
+        pytest.skip("needs a GPU with room for two 66 GiB buffers")
+    n = 65 * G + 12345
+    st = store(66 * G, G)
+    g = torch.Generator(device=DEV)
+    g.manual_seed(65)
+    pat = torch.randint(0, 256, (G,), dtype=torch.uint8, device=DEV, generator=g)
+    x = torch.empty(n, dtype=torch.uint8, device=DEV)
+    for i in range(66):
+        lo, hi = i * G, min((i + 1) * G, n)
+        x[lo:hi] = pat[:hi - lo] ^ (i % 251)
+    s, (oid,) = st.put_batch(put_descs([x]))
+    assert s == 0
+    x.zero_()
+    assert st.get_batch(get_descs([int(oid)], [x]))[0] == 0
+    torch.cuda.synchronize()
+    for i in range(66):
+        lo, hi = i * G, min((i + 1) * G, n)
+        assert torch.equal(x[lo:hi], pat[:hi - lo] ^ (i % 251)), i
+    del x

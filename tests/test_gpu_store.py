@@ -98,12 +98,16 @@ def test_tiny_config_bit_exact():
     assert st.stats()["live_objects"] == 30
 
 
-@pytest.mark.parametrize("seed,P,pages", [(0, 256, 64), (1, 4096, 48), (2, 64 * 1024, 24), (3, 2 * 1024 * 1024, 6),
-                                          (4, 32 * 1024, 40), (5, 1024, 200)])
-def test_random_ops_vs_oracle(seed, P, pages):
+@pytest.mark.parametrize("seed,P,pages,policy", [(0, 256, 64, 0), (1, 4096, 48, 0), (2, 64 * 1024, 24, 0),
+                                                 (3, 2 * 1024 * 1024, 6, 0), (4, 32 * 1024, 40, 0), (5, 1024, 200, 0),
+                                                 (6, 256, 64, 1), (7, 4096, 48, 1), (8, 64 * 1024, 24, 1)])
+def test_random_ops_vs_oracle(seed, P, pages, policy):
+    """Random puts (evictions included), gets, frees and compactions: every
+    status, id, eviction, page list and byte equal to the oracle's, under
+    both placement policies."""
     rng = np.random.default_rng(seed)
-    st = make_store(pages * P, P)
-    ora = OracleStore(pages * P, P)
+    st = make_store(pages * P, P, alloc_policy=policy)
+    ora = OracleStore(pages * P, P, policy=policy)
     keep = []
     for step in range(60):
         r = rng.random()
