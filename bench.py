@@ -402,11 +402,16 @@ class Dist:
             import torch.distributed as dist
             self.dist = dist
             self.backend = backend or ("nccl" if torch.cuda.is_available() else "gloo")
+            if self.backend == "nccl":
+                torch.cuda.set_device(self.local)   # each rank's collectives on its own GPU
             dist.init_process_group(self.backend)
 
     def barrier(self):
         if self.on:
-            self.dist.barrier()
+            if self.backend == "nccl":
+                self.dist.barrier(device_ids=[self.local])
+            else:
+                self.dist.barrier()
 
     def _reduce(self, x: float, op) -> float:
         if not self.on:
