@@ -515,12 +515,15 @@ def test_handoff_spread_over_streams():
     assert st.stats()["used_pages"] == 0
 
 
-def test_bench_step_over_streams():
-    """The benchmark's own multi-stream step (phase joins included) gives
-    get(put(x)) == x and the oracle's cast at B = 1."""
+@pytest.mark.parametrize("B", [1, 8])
+def test_bench_step_over_streams(B):
+    """The benchmark's own multi-stream step (phase joins included), at the
+    headline's size and launch configuration (B = 8, 64 requests, 4 streams)
+    and at B = 1: get(put(x)) == x for every output, the oracle's cast for
+    sampled requests."""
     import bench
 
-    hw = bench.Handoff(1, W.HANDOFF["requests"], DEV)
+    hw = bench.Handoff(B, W.HANDOFF["requests"], DEV)
     streams = [torch.cuda.current_stream()] + [torch.cuda.Stream() for _ in range(3)]
     for _ in range(3):
         hw.step_streams(streams)
