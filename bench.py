@@ -386,6 +386,46 @@ def time_handoff(hw: Handoff, steps: int, warmup: int, dist_ctx, per_kernel: boo
     return ms, launches, kern, (clk.summary() if clk else None)
 
 
+def time_calls(hw: Handoff, reps: int = 3) -> dict:
+    """Each batched call of one step timed alone with CUDA events around it
+    (one stream; an event between two launches keeps the second from
+    starting early, so these are slightly slower than back to back):
+    median and best over the step's 64 puts and 64 gets, ``reps`` times."""
+    torch = hw.torch
+    lib, h, n = hw.lib, hw.h, hw.n_obj
+    stream = torch.cuda.current_stream(hw.device)
+    s = C.c_void_p(stream.cuda_stream)
+    hw.step(stream.cuda_stream)                                     # warm
+    torch.cuda.synchronize(hw.device)
+    put_ms, get_ms = [], []
+    for _ in range(reps):
+        ev = [torch.cuda.Event(enable_timing=True) for _ in range(4 * hw.requests)]
+        for r in range(hw.requests):
+            ev[2 * r].record(stream)
+            if lib.t2i_put_batch(h, hw.pd_p[r], n, hw.ids_p[r], s):
+                raise RuntimeError("put_batch: " + hw.store.last_error())
+            ev[2 * r + 1].record(stream)
+        for r in range(hw.requests):
+            hw.gd[r]["id"] = hw.ids[n * r:n * (r + 1)]
+            k = 2 * hw.requests + 2 * r
+            ev[k].record(stream)
+            if lib.t2i_get_batch(h, hw.gd_p[r], n, None, s):
+                raise RuntimeError("get_batch: " + hw.store.last_error())
+            ev[k + 1].record(stream)
+        torch.cuda.synchronize(hw.device)
+        if lib.t2i_free(h, hw.all_ids_p, len(hw.ids)):
+            raise RuntimeError("free: " + hw.store.last_error())
+        put_ms += [ev[2 * r].elapsed_time(ev[2 * r + 1]) for r in range(hw.requests)]
+        get_ms += [ev[2 * hw.requests + 2 * r].elapsed_time(ev[2 * hw.requests + 2 * r + 1])
+                   for r in range(hw.requests)]
+    pb, gb = hw.put_bytes / hw.requests, hw.get_bytes / hw.requests
+    return {"calls": len(put_ms) + len(get_ms),
+            "put_ms": {"median": round(statistics.median(put_ms), 5), "best": round(min(put_ms), 5)},
+            "get_ms": {"median": round(statistics.median(get_ms), 5), "best": round(min(get_ms), 5)},
+            "put_gbs_median": round(pb / (statistics.median(put_ms) * 1e-3) / 1e9, 1),
+            "get_gbs_median": round(gb / (statistics.median(get_ms) * 1e-3) / 1e9, 1)}
+
+
 class Dist:
     """Rank bookkeeping for N independent replicas (one store per GPU; the
     store has no cross-GPU step, so the only collectives are the timing
@@ -1534,6 +1574,7 @@ def main():
                                   "get_achieved": round(r1["get"], 1), "put_achieved": round(r1["put"], 1),
                                   "get_frac": round(r1["get"] / peak, 4),
                                   "get_avg_launch_ms": round(kern1["get_phase_ms"] / hw.requests, 5)}
+    per_call = time_calls(hw)
     del hw
     torch.cuda.empty_cache()
 
@@ -1648,7 +1689,7 @@ def main():
                        "bytes_per_step": hw_bytes(B, args.requests), "l2": "inputs > L2 (no flush)",
                        "parallelism": f"replicas x{dist_ctx.world}"},
             "hbm_frac": round(value / dist_ctx.world / peak, 4), "hbm_frac_nominal_8tbs": round(value / dist_ctx.world / 8000.0, 4),
-            "step_ms": kern["step_ms"],
+            "step_ms": kern["step_ms"], "per_call": per_call,
             "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e, "gpu_launches": int(launches),
             "clocks": clocks, "sweep": sweep or None, "extras": extras or None, "rows": rows or None,
         }
