@@ -140,3 +140,27 @@ def test_object_larger_than_64_gib():
         lo, hi = i * G, min((i + 1) * G, n)
         assert torch.equal(x[lo:hi], pat[:hi - lo] ^ (i % 251)), i
     del x
+
+
+def test_large_unaligned_launches_take_chunks():
+    """A 400 MiB object put from a source 3 bytes past alignment and got into
+    destinations 5 bytes (copy) and 2 bytes (cast) past it: launches large
+    enough for chunks from the work counter, in the any-alignment kernels."""
+    P = 2 << 20
+    n = 400 << 20
+    st = store(210 * P, P)
+    g = torch.Generator(device=DEV)
+    g.manual_seed(400)
+    f = torch.randn(n // 4, generator=g, device=DEV)
+    src = torch.zeros(n + 16, dtype=torch.uint8, device=DEV)
+    src[3:3 + n] = f.view(torch.uint8)
+    s, (i,) = st.put_batch(put_descs([src.data_ptr() + 3], nbytes=[n]))
+    assert s == 0
+    out = torch.zeros(n + 16, dtype=torch.uint8, device=DEV)
+    assert st.get_batch(get_descs([int(i)], [out.data_ptr() + 5], dst_bytes=[n]))[0] == 0
+    bf = torch.zeros(n // 2 + 16, dtype=torch.uint8, device=DEV)
+    assert st.get_batch(get_descs([int(i)], [bf.data_ptr() + 2], dst_bytes=[n // 2], cast=1))[0] == 0
+    torch.cuda.synchronize()
+    assert torch.equal(out[5:5 + n], f.view(torch.uint8))
+    assert torch.equal(bf[2:2 + n // 2].view(torch.bfloat16), f.to(torch.bfloat16))
+    assert out[:5].sum() == 0 and out[5 + n:].sum() == 0
