@@ -24,7 +24,7 @@ What the store computes, and where the paper fixes it:
   arena problem (§5.3, "Can NVSHMEM region be elastic?") by handing a
   contiguous tail of the pool back.
 
-Readings where the paper is silent (each also listed in the design doc):
+Readings where the paper is silent:
 
 1. Pages: fixed P-byte pages; an object's pages need not be contiguous; the
    unused tail of its last page is never read.
