@@ -62,12 +62,15 @@ _PU32 = C.POINTER(C.c_uint32)
 PROTOTYPES = {
     "t2i_store_create": (_S, [_P, C.POINTER(StoreConfig), C.c_int, C.POINTER(_P)]),
     "t2i_store_destroy": (_S, [_P]),
-    "t2i_put_batch": (_S, [_P, C.POINTER(PutDesc), _U32, _PU64, _P]),
-    "t2i_get_batch": (_S, [_P, C.POINTER(GetDesc), _U32, C.POINTER(_S), _P]),
-    "t2i_get_batch_after": (_S, [_P, C.POINTER(GetDesc), _U32, C.POINTER(_S), _P, _P]),
+    # array arguments of the per-request calls are plain addresses (ints,
+    # numpy buffers' ctypes.data or typed pointers all pass): building a
+    # typed pointer costs more than the call's other Python work
+    "t2i_put_batch": (_S, [_P, _P, _U32, _P, _P]),
+    "t2i_get_batch": (_S, [_P, _P, _U32, _P, _P]),
+    "t2i_get_batch_after": (_S, [_P, _P, _U32, _P, _P, _P]),
     "t2i_view": (_S, [_P, _U64, _P, C.POINTER(_P), _PU64]),
-    "t2i_pull": (_S, [_P, _P, _PU64, _U32, _U32, _PU64, C.POINTER(_S), _P]),
-    "t2i_free": (_S, [_P, _PU64, _U32]),
+    "t2i_pull": (_S, [_P, _P, _P, _U32, _U32, _P, _P, _P]),
+    "t2i_free": (_S, [_P, _P, _U32]),
     "t2i_compact": (_S, [_P, _U64, _P, _PU64]),
     "t2i_inject_launch_failure": (_S, [_P, _U32]),
     "t2i_store_stats": (_S, [_P, C.POINTER(Stats)]),

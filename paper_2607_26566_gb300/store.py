@@ -101,6 +101,14 @@ def _as(arr: np.ndarray, ctype, dtype):
     return arr.ctypes.data_as(C.POINTER(ctype))
 
 
+def _addr(arr: np.ndarray, dtype) -> int:
+    """Address of a descriptor array with the C layout (for the calls that
+    take plain addresses)."""
+    if arr.dtype != dtype or not arr.flags.c_contiguous:
+        raise TypeError("descriptor array has the wrong layout")
+    return arr.ctypes.data
+
+
 class Ctl:
     """The host control core alone (t2i_ctl_*): page allocator, directory,
     LRU and compaction planner without device memory."""
@@ -226,29 +234,60 @@ class Store:
     def put_batch(self, descs: np.ndarray, stream=None):
         """(status, ids) -- t2i_put_batch."""
         ids = np.zeros(len(descs), np.uint64)
-        st = self._lib.t2i_put_batch(self._h, _as(descs, L.PutDesc, PUT_DTYPE), len(descs),
-                                     ids.ctypes.data_as(C.POINTER(C.c_uint64)), _stream(stream))
+        st = self._lib.t2i_put_batch(self._h, _addr(descs, PUT_DTYPE), len(descs), ids.ctypes.data, _stream(stream))
         return st, ids
+
+    # -- prepared batches: descriptors whose buffers stay the same from call
+    #    to call (a serving loop's staging tensors) are checked and converted
+    #    once; each call then passes cached addresses only
+    class Prepared:
+        __slots__ = ("descs", "n", "addr", "out", "out_addr")
+
+        def __init__(self, descs: np.ndarray, dtype, out_dtype):
+            self.descs = descs
+            self.n = len(descs)
+            self.addr = _addr(descs, dtype)
+            self.out = np.zeros(self.n, out_dtype)
+            self.out_addr = self.out.ctypes.data
+
+    def prepare_put(self, descs: np.ndarray) -> "Store.Prepared":
+        """A put batch for :meth:`put_prepared` (the array is kept, not copied)."""
+        return Store.Prepared(descs, PUT_DTYPE, np.uint64)
+
+    def put_prepared(self, p: "Store.Prepared", stream=None):
+        """(status, ids) -- t2i_put_batch on a prepared batch. ``ids`` is the
+        batch's own array, overwritten by the next call."""
+        return self._lib.t2i_put_batch(self._h, p.addr, p.n, p.out_addr, _stream(stream)), p.out
+
+    def prepare_get(self, descs: np.ndarray) -> "Store.Prepared":
+        """A get batch for :meth:`get_prepared` (the array is kept, not copied)."""
+        return Store.Prepared(descs, GET_DTYPE, np.int32)
+
+    def get_prepared(self, p: "Store.Prepared", ids=None, stream=None) -> int:
+        """t2i_get_batch on a prepared batch, after setting its ids to ``ids``
+        (if given); per-item statuses land in ``p.out``."""
+        if ids is not None:
+            p.descs["id"] = ids
+        return self._lib.t2i_get_batch(self._h, p.addr, p.n, p.out_addr, _stream(stream))
 
     def get_batch(self, descs: np.ndarray, stream=None, per_item: bool = True, wait_event=None):
         """(status, per-item statuses) -- t2i_get_batch, or t2i_get_batch_after
         when ``wait_event`` (a torch.cuda.Event or a cudaEvent_t address) is given."""
         per = np.zeros(len(descs), np.int32) if per_item else None
-        per_p = per.ctypes.data_as(C.POINTER(C.c_int32)) if per_item else None
+        per_p = per.ctypes.data if per_item else None
         if wait_event is None:
-            st = self._lib.t2i_get_batch(self._h, _as(descs, L.GetDesc, GET_DTYPE), len(descs), per_p,
-                                         _stream(stream))
+            st = self._lib.t2i_get_batch(self._h, _addr(descs, GET_DTYPE), len(descs), per_p, _stream(stream))
         else:
             ev = wait_event if isinstance(wait_event, int) else int(wait_event.cuda_event)
             if not ev:
                 raise ValueError("wait_event has never been recorded")
-            st = self._lib.t2i_get_batch_after(self._h, _as(descs, L.GetDesc, GET_DTYPE), len(descs), per_p,
+            st = self._lib.t2i_get_batch_after(self._h, _addr(descs, GET_DTYPE), len(descs), per_p,
                                                _stream(stream), ev)
         return st, per
 
     def free(self, ids) -> int:
         ids = np.ascontiguousarray(ids, np.uint64)
-        return self._lib.t2i_free(self._h, ids.ctypes.data_as(C.POINTER(C.c_uint64)), len(ids))
+        return self._lib.t2i_free(self._h, ids.ctypes.data, len(ids))
 
     def pull(self, src: "Store", ids, consumers: int = 0, stream=None):
         """(status, new ids, per-item statuses) -- t2i_pull: this store (the
@@ -256,8 +295,7 @@ class Store:
         ids = np.ascontiguousarray(ids, np.uint64)
         out = np.zeros(len(ids), np.uint64)
         per = np.zeros(len(ids), np.int32)
-        st = self._lib.t2i_pull(self._h, src._h, ids.ctypes.data_as(C.POINTER(C.c_uint64)), len(ids), consumers,
-                                out.ctypes.data_as(C.POINTER(C.c_uint64)), per.ctypes.data_as(C.POINTER(C.c_int32)),
+        st = self._lib.t2i_pull(self._h, src._h, ids.ctypes.data, len(ids), consumers, out.ctypes.data, per.ctypes.data,
                                 _stream(stream))
         return st, out, per
 

@@ -700,3 +700,24 @@ def test_streams_beyond_the_counter_slots_split_statically():
     assert st.get_batch(get_descs([int(i)], [out]), stream=streams[-1])[0] == 0
     torch.cuda.synchronize()
     assert torch.equal(out, x) and torch.equal(small, tiny)
+
+
+def test_prepared_batches():
+    """Prepared put and get batches (descriptors converted once, issued many
+    times) move the same bytes as the plain calls, call after call."""
+    P = 64 * 1024
+    st = make_store(64 * P, P)
+    xs = [torch.randint(0, 256, (n,), dtype=torch.uint8, device=DEV) for n in (5 * P + 3, 100, 2 * P)]
+    outs = [torch.zeros_like(x) for x in xs]
+    pp = st.prepare_put(put_descs(xs))
+    pg = st.prepare_get(get_descs(np.zeros(3, np.uint64), outs))
+    for k in range(3):
+        s, ids = st.put_prepared(pp)
+        assert s == 0
+        assert st.get_prepared(pg, ids) == 0 and list(pg.out) == [0, 0, 0]
+        torch.cuda.synchronize()
+        assert all(torch.equal(o, x) for o, x in zip(outs, xs)), k
+        assert st.free(ids.copy()) == 0
+        for o in outs:
+            o.zero_()
+    assert st.stats()["used_pages"] == 0
