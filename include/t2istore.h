@@ -222,6 +222,36 @@ t2i_status t2i_view(t2i_store* store, t2i_id id, void* cuda_stream, void** dev_p
 t2i_status t2i_pull(t2i_store* dst, t2i_store* src, const t2i_id* src_ids, uint32_t n, uint32_t consumers,
                     t2i_id* out_ids, t2i_status* per_item, void* cuda_stream);
 
+/* One object laid out in pages of a pool that the pulling store does not
+ * own (t2i_pull_pages).                                                     */
+typedef struct {
+    uint64_t nbytes;        /* the object's size in bytes                      */
+    const uint32_t* pages;  /* its page list in byte order: page indices into
+                               the source pool (host array, read during the
+                               call)                                           */
+    uint32_t n_pages;       /* ceil(nbytes / page_bytes)                       */
+    uint32_t dtype_tag;     /* kept on the new object                          */
+} t2i_paged_object;
+
+/* Pulls n objects laid out in pages of another pool into `dst` (§5.2: the
+ * consumer allocates a block in its own arena and pulls the producer's bytes
+ * into it), page to page on the GPU. The source pool is usually a producer
+ * store's pool in another process on the same GPU, mapped into this one with
+ * cudaIpcOpenMemHandle (torch shares CUDA tensors between processes this
+ * way); the page lists come from the producer (t2i_ctl_object).
+ * src_pool: device memory of dst's device covering src_pool_bytes, laid out
+ * in pages of dst's page size, not overlapping dst's pool. Each object's
+ * pages must lie in the source pool and number ceil(nbytes / page_bytes).
+ * out_ids[i] receives the new id of objs[i]: an intermediate (evictable = 0,
+ * group 0, order 0) with objs[i].dtype_tag and `consumers`. NOSPACE in dst
+ * changes nothing. The source is not a store of this process: the caller
+ * orders its bytes before this call (the producer synchronizes, or its event
+ * is waited on), and keeps them until the copy has run on cuda_stream. The
+ * copy is ordered after dst's earlier users of the new pages.               */
+t2i_status t2i_pull_pages(t2i_store* dst, const void* src_pool, uint64_t src_pool_bytes,
+                          const t2i_paged_object* objs, uint32_t n, uint32_t consumers, t2i_id* out_ids,
+                          void* cuda_stream);
+
 /* Returns the pages of n objects to the free stack (paper §5.3: data is
  * reclaimed when no consumer needs it). Host-only: stream order makes reuse
  * safe. A repeated id is INVALID; an unknown id is NOT_FOUND; in both cases

@@ -51,6 +51,10 @@ class ObjectInfo(C.Structure):
                 ("reserved", C.c_uint32)]
 
 
+class PagedObject(C.Structure):
+    _fields_ = [("nbytes", C.c_uint64), ("pages", C.c_void_p), ("n_pages", C.c_uint32), ("dtype_tag", C.c_uint32)]
+
+
 _P = C.c_void_p
 _S = C.c_int32
 _U32 = C.c_uint32
@@ -70,6 +74,7 @@ PROTOTYPES = {
     "t2i_get_batch_after": (_S, [_P, _P, _U32, _P, _P, _P]),
     "t2i_view": (_S, [_P, _U64, _P, C.POINTER(_P), _PU64]),
     "t2i_pull": (_S, [_P, _P, _P, _U32, _U32, _P, _P, _P]),
+    "t2i_pull_pages": (_S, [_P, _P, _U64, _P, _U32, _U32, _P, _P]),
     "t2i_free": (_S, [_P, _P, _U32]),
     "t2i_compact": (_S, [_P, _U64, _P, _PU64]),
     "t2i_inject_launch_failure": (_S, [_P, _U32]),

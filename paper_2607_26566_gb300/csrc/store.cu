@@ -186,6 +186,8 @@ class Store {
     t2i_status view(t2i_id id, cudaStream_t stream, void** ptr, uint64_t* nbytes);
     t2i_status pull_from(Store& src, const t2i_id* ids, uint32_t n, uint32_t consumers, t2i_id* out_ids,
                          t2i_status* per_item, cudaStream_t stream);
+    t2i_status pull_pages(const void* src_pool, uint64_t src_pool_bytes, const t2i_paged_object* objs, uint32_t n,
+                          uint32_t consumers, t2i_id* out_ids, cudaStream_t stream);
 
   private:
     // ---- pointer checks (per call cache of the last allocation seen)
@@ -637,6 +639,90 @@ t2i_status Store::pull_from(Store& src, const t2i_id* ids, uint32_t n, uint32_t 
     return st;
 }
 
+// The consumer's half of a pull whose producer is not a store of this
+// process: the source pages are given as a pool address and page lists.
+t2i_status Store::pull_pages(const void* src_pool, uint64_t src_pool_bytes, const t2i_paged_object* objs, uint32_t n,
+                             uint32_t consumers, t2i_id* out_ids, cudaStream_t stream) {
+    if (n == 0) return T2I_OK;
+    if (!src_pool || !objs || !out_ids) {
+        err_ = "pull_pages: null pool, object or id array";
+        return T2I_ERR_INVALID;
+    }
+    const uint64_t P = uint64_t(1) << page_shift_;
+    const uint64_t sp = reinterpret_cast<uint64_t>(src_pool);
+    if (src_pool_bytes < P || sp % 256 != 0 || sp + src_pool_bytes < sp) {
+        err_ = "pull_pages: the source pool must be 256-byte aligned and hold at least one page";
+        return T2I_ERR_INVALID;
+    }
+    if (overlaps_pool(sp, src_pool_bytes)) {
+        err_ = "pull_pages: the source pool overlaps this store's pool";
+        return T2I_ERR_INVALID;
+    }
+    Range r;
+    if (!query_range(src_pool, &r) || r.kind != MemKind::Device || r.device != device_ || sp + src_pool_bytes > r.end) {
+        err_ = "pull_pages: the source pool must be device memory of this store's device covering src_pool_bytes";
+        return T2I_ERR_INVALID;
+    }
+    // 1. every object's page list first (a failed pull changes nothing)
+    const uint64_t src_pages = src_pool_bytes / P;
+    for (uint32_t i = 0; i < n; ++i) {
+        const t2i_paged_object& o = objs[i];
+        if (o.n_pages != o.nbytes / P + (o.nbytes % P != 0) || (o.n_pages && !o.pages)) {
+            err_ = "pull_pages: object " + std::to_string(i) + ": n_pages must be nbytes / page_bytes rounded up";
+            return T2I_ERR_INVALID;
+        }
+        for (uint32_t j = 0; j < o.n_pages; ++j)
+            if (o.pages[j] >= src_pages) {
+                err_ = "pull_pages: object " + std::to_string(i) + ": a page lies outside the source pool";
+                return T2I_ERR_INVALID;
+            }
+    }
+    // 2. room in this store, as intermediates
+    std::vector<t2i_put_desc> pd(n);
+    for (uint32_t i = 0; i < n; ++i) pd[i] = t2i_put_desc{nullptr, objs[i].nbytes, 0, objs[i].dtype_tag, 0, 0, 0, consumers, 0};
+    t2i_status st = ctl_.put(pd.data(), n, out_ids, &objs_);
+    if (st != T2I_OK) {
+        err_ = ctl_.error();
+        return st;
+    }
+    // 3. page-to-page copies, after this store's earlier users of the new pages
+    DeviceGuard g(device_);
+    int si = 0;
+    if ((st = stream_slot(stream, &si)) != T2I_OK) {
+        ctl_.rollback_put(out_ids, n);
+        return st;
+    }
+    deps_.begin(si);
+    segs_.clear();
+    for (uint32_t i = 0; i < n; ++i) {
+        const Object* d_o = objs_[i];
+        for (uint32_t j = 0; j < objs[i].n_pages; ++j) {
+            deps_.writes(d_o->pages[j]);
+            segs_.push_back({sp + uint64_t(objs[i].pages[j]) * P, std::min<uint64_t>(P, objs[i].nbytes - uint64_t(j) * P),
+                             &d_o->pages[j], 1u});
+        }
+    }
+    if (segs_.empty()) return T2I_OK;
+    cudaError_t we = deps_.wait();
+    if (we != cudaSuccess) {
+        ctl_.rollback_put(out_ids, n);
+        return cuda_fail("pull_pages: cannot order after earlier calls", we);
+    }
+    st = launch_segments<Mode::Move>(segs_, stream);
+    // marked even after a failure part-way: launches before it may still be
+    // writing the pages handed back
+    uint32_t q = 0;
+    cudaError_t ee = deps_.end(&q);
+    for (uint32_t i = 0; i < n; ++i)
+        for (uint32_t pg : objs_[i]->pages) deps_.mark_write(pg, q);
+    if (st != T2I_OK) {
+        ctl_.rollback_put(out_ids, n);
+        return st;
+    }
+    if (ee != cudaSuccess) return cuda_fail("pull_pages: cannot record its event", ee);
+    return T2I_OK;
+}
+
 t2i_status Store::compact(uint64_t limit_bytes, cudaStream_t stream, uint64_t* moved) {
     if (moved) *moved = 0;
     t2i_status st = ctl_.begin_compact(limit_bytes);
@@ -865,6 +951,13 @@ t2i_status t2i_pull(t2i_store* dst, t2i_store* src, const t2i_id* src_ids, uint3
         dst->s->set_error(std::string("host error: ") + e.what());
         return T2I_ERR_INVALID;
     }
+}
+
+t2i_status t2i_pull_pages(t2i_store* dst, const void* src_pool, uint64_t src_pool_bytes,
+                          const t2i_paged_object* objs, uint32_t n, uint32_t consumers, t2i_id* out_ids,
+                          void* cuda_stream) {
+    T2I_STORE_CALL(dst, dst->s->pull_pages(src_pool, src_pool_bytes, objs, n, consumers, out_ids,
+                                          static_cast<cudaStream_t>(cuda_stream)));
 }
 
 t2i_status t2i_compact(t2i_store* store, uint64_t limit_bytes, void* cuda_stream, uint64_t* pages_moved) {

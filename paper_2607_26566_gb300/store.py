@@ -289,6 +289,22 @@ class Store:
         ids = np.ascontiguousarray(ids, np.uint64)
         return self._lib.t2i_free(self._h, ids.ctypes.data, len(ids))
 
+    def pull_pages(self, src_pool, objects, src_pool_bytes: int | None = None, consumers: int = 0, stream=None):
+        """(status, new ids) -- t2i_pull_pages: pulls objects laid out in pages
+        of another pool (e.g. a producer store's pool shared from another
+        process). ``objects``: (nbytes, page list, dtype_tag) triples."""
+        objs = (L.PagedObject * max(1, len(objects)))()
+        keep = []
+        for i, (nbytes, pages, tag) in enumerate(objects):
+            pg = np.ascontiguousarray(pages, np.uint32)
+            keep.append(pg)
+            objs[i] = L.PagedObject(int(nbytes), pg.ctypes.data if len(pg) else None, len(pg), int(tag))
+        out = np.zeros(len(objects), np.uint64)
+        nb = src_pool_bytes if src_pool_bytes is not None else _nbytes(src_pool)
+        st = self._lib.t2i_pull_pages(self._h, _ptr(src_pool), int(nb), C.addressof(objs), len(objects), consumers,
+                                      out.ctypes.data, _stream(stream))
+        return st, out
+
     def pull(self, src: "Store", ids, consumers: int = 0, stream=None):
         """(status, new ids, per-item statuses) -- t2i_pull: this store (the
         consumer) pulls ``ids`` from the producer's store ``src``."""

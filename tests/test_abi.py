@@ -52,6 +52,7 @@ int main(void) {
   printf("%zu %zu %zu %zu %zu %zu\\n", sizeof(t2i_store_config), sizeof(t2i_put_desc), sizeof(t2i_get_desc),
          sizeof(t2i_move), sizeof(t2i_stats), sizeof(t2i_object_info));
   printf("%zu %zu %zu\\n", offsetof(t2i_put_desc, group), offsetof(t2i_get_desc, cast), offsetof(t2i_move, valid_bytes));
+  printf("%zu %zu\\n", sizeof(t2i_paged_object), offsetof(t2i_paged_object, n_pages));
   return 0;
 }
 """)
@@ -61,7 +62,8 @@ int main(void) {
     out = subprocess.run([str(exe)], capture_output=True, text=True, check=True).stdout.split()
     got = [int(x) for x in out]
     want = [C.sizeof(L.StoreConfig), C.sizeof(L.PutDesc), C.sizeof(L.GetDesc), C.sizeof(L.Move), C.sizeof(L.Stats),
-            C.sizeof(L.ObjectInfo), L.PutDesc.group.offset, L.GetDesc.cast.offset, L.Move.valid_bytes.offset]
+            C.sizeof(L.ObjectInfo), L.PutDesc.group.offset, L.GetDesc.cast.offset, L.Move.valid_bytes.offset,
+            C.sizeof(L.PagedObject), L.PagedObject.n_pages.offset]
     assert got == want
 
 
