@@ -1312,6 +1312,112 @@ def time_pull(device, B: int = 8, requests: int = 64, reps: int = 3):
     return res
 
 
+def _ipc_producer(to_parent, from_parent, B: int, requests: int, seed: int, device_index: int):
+    """A producer executor in its own process: puts the handoff requests into
+    its store and shares the pool (CUDA IPC, through torch) and the page
+    lists with the consumer, until the consumer is done."""
+    import torch
+
+    from paper_2607_26566_gb300 import Store, put_descs
+
+    dev = torch.device("cuda", device_index)
+    torch.cuda.set_device(dev)
+    specs = W.handoff_specs(B)
+    pool = torch.empty(W.HANDOFF["pool_bytes"], dtype=torch.uint8, device=dev)
+    st = Store(pool, W.HANDOFF["page_bytes"])
+    objects = []
+    for r in range(requests):
+        ts = W.handoff_request_torch(seed, r, specs, dev)
+        s, ids = st.put_batch(put_descs(ts, nbytes=[sp.nbytes for sp in specs]))
+        st.check(s)
+        objects.append([(sp.nbytes, st.ctl.object(int(i))[2], sp.dtype_tag) for sp, i in zip(specs, ids)])
+        torch.cuda.synchronize(dev)
+        del ts
+    to_parent.put((pool, objects))
+    from_parent.get(timeout=600)
+    st.close()
+
+
+def time_pull_ipc(device, B: int = 8, requests: int = 64, reps: int = 3, n_streams: int = 4, seed: int = 5):
+    """The handoff pulled across processes: a spawned producer shares its
+    store's pool through CUDA IPC, and this process pulls every request into
+    its own store with t2i_pull_pages, request r on stream r % n_streams."""
+    import torch
+    import torch.multiprocessing as tmp
+
+    from paper_2607_26566_gb300 import Store, get_descs
+    from paper_2607_26566_gb300 import _lib as L
+
+    ctx = tmp.get_context("spawn")
+    to_parent, from_parent = ctx.Queue(), ctx.Queue()
+    child = ctx.Process(target=_ipc_producer, args=(to_parent, from_parent, B, requests, seed, device.index or 0))
+    child.start()
+    try:
+        src_pool, objects = to_parent.get(timeout=600)
+        cons = Store(torch.empty(W.HANDOFF["pool_bytes"], dtype=torch.uint8, device=device), W.HANDOFF["page_bytes"])
+        lib = cons._lib
+        # C arrays built once: each pull is a raw C-ABI call
+        keep, arrays = [], []
+        for objs in objects:
+            arr = (L.PagedObject * len(objs))()
+            for j, (nb, pages, tag) in enumerate(objs):
+                pg = np.ascontiguousarray(pages, np.uint32)
+                keep.append(pg)
+                arr[j] = L.PagedObject(int(nb), pg.ctypes.data, len(pg), int(tag))
+            arrays.append(arr)
+        n = len(objects[0])
+        new = np.zeros(requests * n, np.uint64)
+        streams = [torch.cuda.current_stream(device)] + [torch.cuda.Stream(device) for _ in range(n_streams - 1)]
+        ss = [C.c_void_p(x.cuda_stream) for x in streams]
+        sp, spb = src_pool.data_ptr(), src_pool.numel()
+
+        def once():
+            for r in range(requests):
+                st = lib.t2i_pull_pages(cons._h, sp, spb, C.addressof(arrays[r]), n, 0,
+                                        new.ctypes.data + 8 * n * r, ss[r % n_streams])
+                if st:
+                    raise RuntimeError("pull_pages: " + cons.last_error())
+            cons.check(cons.free(new))
+
+        once()
+        torch.cuda.synchronize(device)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(streams[0])
+        for x in streams[1:]:
+            x.wait_event(e0)
+        for _ in range(reps):
+            once()
+        for x in streams[1:]:
+            ev = torch.cuda.Event()
+            ev.record(x)
+            streams[0].wait_event(ev)
+        e1.record(streams[0])
+        torch.cuda.synchronize(device)
+        ms = e0.elapsed_time(e1) / reps
+        payload = sum(nb for objs in objects for nb, _, _ in objs)
+        # request 0 pulled once more and compared with its inputs
+        s, ids = cons.pull_pages(src_pool, objects[0])
+        cons.check(s)
+        specs = W.handoff_specs(B)
+        want = W.handoff_request_torch(seed, 0, specs, device)
+        outs = [torch.empty(sp.nbytes, dtype=torch.uint8, device=device) for sp in specs]
+        cons.check(cons.get_batch(get_descs(ids, outs), per_item=False)[0])
+        torch.cuda.synchronize(device)
+        ok = all(torch.equal(t.reshape(-1).view(torch.uint8), o) for t, o in zip(want, outs))
+        res = {"ipc_workload": f"the {requests} B={B} requests pulled from a producer process's store (CUDA IPC), "
+                               f"{n_streams} streams",
+               "ipc_ms": round(ms, 3), "ipc_gbs": round(2 * payload / (ms * 1e-3) / 1e9, 1), "ipc_bit_exact": bool(ok)}
+        cons.close()
+        del src_pool
+        from_parent.put("done")
+        child.join(timeout=120)
+        return res
+    finally:
+        if child.is_alive():
+            child.terminate()
+            child.join(timeout=30)
+
+
 # ----------------------------------------------------------------------------- CPU (oracle)
 def oracle_sample(B: int, n_requests: int, min_seconds: float = 0.0, max_steps: int = 1):
     """The oracle as it stands on the host: steps of the handoff workload (put
@@ -1508,6 +1614,10 @@ def run_rows(args, device, peak):
         rows["views"] = time_views(device)
     if "pull" in wanted:
         rows["pull"] = time_pull(device)
+        try:
+            rows["pull"].update(time_pull_ipc(device))
+        except Exception as e:  # a box without CUDA IPC: the same-process row stands
+            rows["pull"]["ipc_error"] = f"{type(e).__name__}: {e}"
     for r in rows.values():
         for k in ("get_gbs", "gbs", "hit_gbs"):
             if k in r:

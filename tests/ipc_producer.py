@@ -1,11 +1,12 @@
-"""The producer process of the cross-process pull test (imported by the
-spawned child; not a test module): it puts objects into its own store,
-shares the store's pool with the parent through CUDA IPC (torch sends CUDA
-tensors between processes that way) together with the objects' page lists
-and expected bytes, and keeps the pool alive until the parent is done."""
+"""Producer processes for cross-process pulls (imported by spawned children;
+not a test module). A producer puts objects into its own store, shares the
+store's pool with the parent through CUDA IPC (torch sends CUDA tensors
+between processes that way) together with the objects' page lists, and keeps
+the pool alive until the parent is done with it."""
 
 
 def run(to_parent, from_parent, sizes, page_bytes, seed):
+    """Objects of ``sizes`` bytes; also sends their expected bytes."""
     import torch
 
     from paper_2607_26566_gb300 import Store, put_descs
