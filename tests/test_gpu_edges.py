@@ -164,3 +164,36 @@ def test_large_unaligned_launches_take_chunks():
     assert torch.equal(out[5:5 + n], f.view(torch.uint8))
     assert torch.equal(bf[2:2 + n // 2].view(torch.bfloat16), f.to(torch.bfloat16))
     assert out[:5].sum() == 0 and out[5 + n:].sum() == 0
+
+
+@pytest.mark.parametrize("P", [256, 1024, 4096, 16384])
+def test_small_page_rounds(P):
+    """Objects spanning many pages smaller than a copy round: rounds that
+    cover several pages in put, get, get with a cast in the same launch, and
+    the any-alignment kernels (a source 3 bytes past alignment); every byte
+    against the oracle's get."""
+    rng = np.random.default_rng(P)
+    n_pages = (6 << 20) // P
+    st = store(n_pages * P, P)
+    ora = OracleStore(n_pages * P, P)
+    sizes = [(1 << 20) + 48, 256 * 1024 - 32, (512 << 10) + 4 * 7]
+    datas = [rng.integers(0, 256, n, dtype=np.uint8) for n in sizes]
+    datas[2] = rng.standard_normal(sizes[2] // 4).astype(np.float32).view(np.uint8)
+    srcs = [torch.from_numpy(d).to(DEV) for d in datas]
+    raw = torch.zeros(sizes[0] + 16, dtype=torch.uint8, device=DEV)
+    raw[3:3 + sizes[0]] = srcs[0]
+    s, ids = st.put_batch(put_descs([raw.data_ptr() + 3, srcs[1], srcs[2]], nbytes=sizes))
+    assert s == 0
+    _, oids = ora.put_batch([PutItem(n, d) for n, d in zip(sizes, datas)])
+    assert list(ids) == oids
+    outs = [torch.zeros(sizes[0], dtype=torch.uint8, device=DEV), torch.zeros(sizes[1], dtype=torch.uint8, device=DEV),
+            torch.zeros(sizes[2] // 2, dtype=torch.uint8, device=DEV)]
+    assert st.get_batch(get_descs(ids, outs, dst_bytes=[sizes[0], sizes[1], sizes[2] // 2], cast=[0, 0, 1]))[0] == 0
+    plain = [torch.zeros(n, dtype=torch.uint8, device=DEV) for n in sizes]
+    assert st.get_batch(get_descs(ids, plain))[0] == 0
+    torch.cuda.synchronize()
+    _, _, want = ora.get_batch(oids, [0, 0, 1])
+    for o, w in zip(outs, want):
+        assert np.array_equal(o.cpu().numpy(), w)
+    for o, d in zip(plain, datas):
+        assert np.array_equal(o.cpu().numpy(), d)
