@@ -161,7 +161,8 @@ class Handoff:
     once; a step issues raw C-ABI calls only."""
 
     def __init__(self, B: int, requests: int, device, host_buffers: bool = False, seed: int = 0,
-                 pool_bytes: int | None = None, consumers: int = 0, h2d_mode: int = 0, page_bytes: int | None = None):
+                 pool_bytes: int | None = None, consumers: int = 0, h2d_mode: int = 0, page_bytes: int | None = None,
+                 alloc_policy: int = 0):
         import torch
 
         from paper_2607_26566_gb300 import Store, get_descs, put_descs
@@ -174,7 +175,7 @@ class Handoff:
         self.requests = requests
         self.ci = W.handoff_cast_index()
         self.pool = torch.empty(pool_bytes or C_["pool_bytes"], dtype=torch.uint8, device=device)
-        self.store = Store(self.pool, page_bytes or C_["page_bytes"], h2d_mode=h2d_mode)
+        self.store = Store(self.pool, page_bytes or C_["page_bytes"], h2d_mode=h2d_mode, alloc_policy=alloc_policy)
         self.lib = self.store._lib
         self.h = self.store._h
         self.inputs, self.outputs = [], []

@@ -83,6 +83,10 @@ struct SegDesc {
 };
 static_assert(sizeof(SegDesc) == 24, "SegDesc layout");
 constexpr uint64_t kCastFlag = uint64_t(1) << 63;
+// The segment's pages are consecutive in the pool: its page list holds the
+// first page only, and pieces may cross page boundaries.
+constexpr uint64_t kRunFlag = uint64_t(1) << 62;
+constexpr uint64_t kSegBytesMask = ~(kCastFlag | kRunFlag);
 
 struct LaunchHeader {
     uint64_t pool;            // pool base address (device)
@@ -449,7 +453,7 @@ __device__ __forceinline__ void run_range(const LaunchParams<BLOB>& p, uint64_t 
     // the current segment and page stay in registers until the walk leaves them
     SegDesc s = segs[i];
     uint64_t lo = uint64_t(s.start) * kGranule;
-    uint64_t nbytes = s.nbytes_flags & ~kCastFlag;
+    uint64_t nbytes = s.nbytes_flags & kSegBytesMask;
     uint64_t page_idx = ~uint64_t(0);
     unsigned char* page_base = nullptr;
 #pragma unroll 1
@@ -458,7 +462,7 @@ __device__ __forceinline__ void run_range(const LaunchParams<BLOB>& p, uint64_t 
             if (++i >= p.h.n_seg) break;
             s = segs[i];
             lo = uint64_t(s.start) * kGranule;  // segments are ordered: this is >= pos
-            nbytes = s.nbytes_flags & ~kCastFlag;
+            nbytes = s.nbytes_flags & kSegBytesMask;
             page_idx = ~uint64_t(0);
             pos = lo;
             continue;
@@ -469,19 +473,27 @@ __device__ __forceinline__ void run_range(const LaunchParams<BLOB>& p, uint64_t 
         // stopping at every page end (+2% on a handoff in 16 and 64 KiB pages)
         constexpr uint64_t kRound = uint64_t(kThreads) * kV * 16;
         if (pmask + 1 < kRound && off + kRound <= nbytes && pos + kRound <= end &&
-            !(M == Mode::Get && (s.nbytes_flags & kCastFlag)) &&
+            !(s.nbytes_flags & (kCastFlag | kRunFlag)) &&
             (!GENERAL || (reinterpret_cast<uintptr_t>(s.user) & 15u) == 0)) {
             cta_copy_pages<M, kV>(reinterpret_cast<unsigned char*>(s.user), pool, pages + s.page_begin, off, pshift);
             pos += kRound;
             continue;
         }
-        const uint64_t in_page = off & pmask;
-        if ((off >> pshift) != page_idx) {
-            page_idx = off >> pshift;
-            page_base = pool + (uint64_t(pages[s.page_begin + page_idx]) << pshift);
+        uint32_t len;
+        unsigned char* paddr;
+        if (s.nbytes_flags & kRunFlag) {
+            // consecutive pages: one contiguous stretch of the pool
+            paddr = pool + (uint64_t(pages[s.page_begin]) << pshift) + off;
+            len = (uint32_t)umin64(umin64(end - pos, nbytes - off), kPieceBytes);
+        } else {
+            const uint64_t in_page = off & pmask;
+            if ((off >> pshift) != page_idx) {
+                page_idx = off >> pshift;
+                page_base = pool + (uint64_t(pages[s.page_begin + page_idx]) << pshift);
+            }
+            len = (uint32_t)umin64(umin64(end - pos, nbytes - off), umin64(piece, pmask + 1 - in_page));
+            paddr = page_base + in_page;
         }
-        const uint32_t len = (uint32_t)umin64(umin64(end - pos, nbytes - off), umin64(piece, pmask + 1 - in_page));
-        unsigned char* paddr = page_base + in_page;
         unsigned char* uaddr = reinterpret_cast<unsigned char*>(s.user);
         if (M == Mode::Get || M == Mode::GetCopy) {
             if (M == Mode::Get && (s.nbytes_flags & kCastFlag)) {

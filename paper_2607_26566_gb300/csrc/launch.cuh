@@ -119,14 +119,19 @@ t2i_status Store::launch_group(const std::vector<Seg>& segs, cudaStream_t stream
     const uint64_t max_pages_per_seg = std::min<uint64_t>((kBlobLarge - sizeof(SegDesc)) / sizeof(uint32_t),
                                                           std::max<uint64_t>(1, kMaxSegBytes / P));
     for (const Seg& s : segs) {
-        const uint64_t nbytes = s.nbytes_flags & ~kCastFlag;
+        const uint64_t nbytes = s.nbytes_flags & kSegBytesMask;
         const uint64_t flags = s.nbytes_flags & kCastFlag;
-        for (uint64_t p0 = 0; p0 < s.n_pages; p0 += max_pages_per_seg) {
-            const uint64_t np = std::min<uint64_t>(max_pages_per_seg, s.n_pages - p0);
+        // consecutive pages travel as their first page alone
+        bool run = s.n_pages > 1;
+        for (uint32_t k = 1; run && k < s.n_pages; ++k) run = s.pages[k] == s.pages[0] + k;
+        const uint64_t seg_pages = run ? std::max<uint64_t>(1, kMaxSegBytes / P) : max_pages_per_seg;
+        for (uint64_t p0 = 0; p0 < s.n_pages; p0 += seg_pages) {
+            const uint64_t np = std::min<uint64_t>(seg_pages, s.n_pages - p0);
+            const uint64_t entries = run ? 1 : np;
             const uint64_t off = p0 * P;
             const uint64_t seg_bytes = std::min<uint64_t>(nbytes - off, np * P);
             const uint64_t seg_gran = (seg_bytes + kGranule - 1) / kGranule;
-            const size_t need = (sd_.size() + 1) * sizeof(SegDesc) + (lp_.size() + np) * sizeof(uint32_t);
+            const size_t need = (sd_.size() + 1) * sizeof(SegDesc) + (lp_.size() + entries) * sizeof(uint32_t);
             if (need > size_t(kBlobLarge) || gran + seg_gran > 0xFFFFFFFFull) {
                 t2i_status st = flush();
                 if (st != T2I_OK) return st;
@@ -134,11 +139,11 @@ t2i_status Store::launch_group(const std::vector<Seg>& segs, cudaStream_t stream
             SegDesc d;
             // a get with the cast writes half as many bytes as it reads
             d.user = s.user + (flags ? off / 2 : off);
-            d.nbytes_flags = seg_bytes | flags;
+            d.nbytes_flags = seg_bytes | flags | (run && np > 1 ? kRunFlag : 0);
             d.start = static_cast<uint32_t>(gran);
             d.page_begin = static_cast<uint32_t>(lp_.size());
             sd_.push_back(d);
-            lp_.insert(lp_.end(), s.pages + p0, s.pages + p0 + np);
+            lp_.insert(lp_.end(), s.pages + p0, s.pages + p0 + entries);
             gran += seg_gran;
         }
     }

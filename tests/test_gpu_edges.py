@@ -25,15 +25,27 @@ def store(pool_bytes, page_bytes, **kw):
 
 
 def test_object_longer_than_one_launch():
-    """8,000 pages of 256 B: the page list is split across launches."""
+    """8,000 pages of 256 B in descending order (LIFO reuse): the page list
+    is split across launches. On a fresh store the same object's pages are
+    consecutive and travel as one run, in one launch."""
     P = 256
     st = store(9000 * P, P)
     x = torch.randint(0, 256, (8000 * P - 77,), dtype=torch.uint8, device=DEV)
     s, (i,) = st.put_batch(put_descs([x]))
-    assert s == 0 and st.stats()["launches"] >= 2
+    assert s == 0 and st.stats()["launches"] == 1 and st.ctl.object(int(i))[2] == list(range(8000))
     out = torch.zeros_like(x)
+    assert st.get_batch(get_descs([int(i)], [out]))[0] == 0 and st.stats()["launches"] == 2
+    torch.cuda.synchronize()
+    assert torch.equal(out, x)
+    assert st.free([int(i)]) == 0
+    # the freed pages pop back in descending order: no run
     l0 = st.stats()["launches"]
-    assert st.get_batch(get_descs([int(i)], [out]))[0] == 0
+    s, (j,) = st.put_batch(put_descs([x]))
+    assert s == 0 and st.ctl.object(int(j))[2] == list(range(7999, -1, -1))
+    assert st.stats()["launches"] - l0 >= 2
+    out.zero_()
+    l0 = st.stats()["launches"]
+    assert st.get_batch(get_descs([int(j)], [out]))[0] == 0
     assert st.stats()["launches"] - l0 >= 2
     torch.cuda.synchronize()
     assert torch.equal(out, x)

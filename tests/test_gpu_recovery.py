@@ -128,13 +128,17 @@ def test_failed_put_still_orders_the_pages_it_hands_back():
     s1, s2 = torch.cuda.Stream(), torch.cuda.Stream()
     a = torch.randint(0, 256, (8000 * P,), dtype=torch.uint8, device=DEV)
     b = torch.randint(0, 256, (8000 * P,), dtype=torch.uint8, device=DEV)
+    # a put and a free first: the pages then pop in descending order, so the
+    # object's page list is not one run and takes two launches
+    s, (k,) = st.put_batch(put_descs([a]), stream=s1)
+    assert s == 0 and st.free([int(k)]) == 0
     torch.cuda.synchronize()
     _late(s1, 30)
-    assert st.inject_launch_failure(2) == 0          # 8,000 pages take two launches
+    assert st.inject_launch_failure(2) == 0          # 8,000 scattered pages take two launches
     s, _ = st.put_batch(put_descs([a]), stream=s1)
     assert s == CUDA and st.stats()["used_pages"] == 0
     s, (j,) = st.put_batch(put_descs([b]), stream=s2)
-    assert s == 0 and st.ctl.object(int(j))[2] == list(range(8000))   # the same pages
+    assert s == 0 and st.ctl.object(int(j))[2] == list(range(7999, -1, -1))   # the same pages
     out = torch.zeros_like(b)
     assert st.get_batch(get_descs([int(j)], [out]), stream=s2)[0] == 0
     torch.cuda.synchronize()
