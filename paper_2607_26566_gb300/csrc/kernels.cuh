@@ -17,9 +17,11 @@
 //     share, and the hardware block scheduler hands CTAs to whichever SMs
 //     free up first.
 // Both leave all CTAs finishing within a chunk or a share of each other. A
-// CTA walks its part in pieces of at most U = 32 KiB that lie in one page of
-// one segment, mapping each piece to its page through the segment's page
-// list.
+// CTA walks its part in pieces of at most U = 32 KiB within one segment,
+// mapping each piece to its page through the segment's page list: a piece
+// stays in one page, unless the segment is a run of consecutive pages (then
+// only its first page is listed), and with pages smaller than U one round
+// of the copy covers several pages, each vector finding its own.
 //
 // HBM-bound by construction (2 bytes of traffic per payload byte, 1.5 for the
 // cast): fully coalesced 16-byte accesses, enough bytes in flight per SM (8
@@ -27,9 +29,9 @@
 // CTAs of 256 threads per SM: 96-128 KiB in flight), grids sized from the SM
 // count, the occupancy and the launch's bytes (see the work split above), and
 // programmatic dependent launch so that the next launch's set-up overlaps the
-// end of this one. The launch shape
-// and cache policy were chosen by a sweep on GB300 (default caching beat
-// streaming hints by ~1.5%; 8 vectors per thread beat 2 and 4).
+// end of this one. The launch shape and cache policy were chosen by a sweep
+// on GB300 (default caching beat streaming hints by ~1.5%; 8 vectors per
+// thread beat 2 and 4).
 #pragma once
 
 #include <cstdint>
