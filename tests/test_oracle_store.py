@@ -212,7 +212,7 @@ def test_lru_reverse_layer_hand_trace():
     st, per, _ = s.get_batch([4, 99, 1])
     assert st == EVICTED and per == [EVICTED, NOT_FOUND, OK]
     st, (y,) = s.put_batch([PutItem(P, np.zeros(P, np.uint8), group=2, order=0, evictable=True)])
-    assert st == OK and s.last_evictions == [3]      # group 2 is pinned by this put; layer 2 of model 1
+    assert st == OK and s.last_evictions == [3]      # layer 2 of model 1, now the only evictable model
     assert s.pages_of(y) == [2]
     before = sorted(s.objects)
     st, _ = s.put_batch([PutItem(4 * P, np.zeros(4 * P, np.uint8), group=4)])
@@ -222,6 +222,12 @@ def test_lru_reverse_layer_hand_trace():
     s2.put_batch([PutItem(P, np.zeros(P, np.uint8), group=5, order=1, evictable=True) for _ in range(2)])
     st, _ = s2.put_batch([PutItem(P, np.zeros(P, np.uint8), group=6)])
     assert st == OK and s2.last_evictions == [2]
+    # a put's own groups are never victims, even when they are the least recent
+    s3 = OracleStore(3 * P, P)
+    s3.put_batch([PutItem(P, None, group=7, evictable=True)])
+    _, (b3, c3) = s3.put_batch([PutItem(P, None, group=8, order=k, evictable=True) for k in range(2)])
+    st, _ = s3.put_batch([PutItem(P, None, group=7, order=1, evictable=True)])
+    assert st == OK and s3.last_evictions == [c3]    # model 8's last layer, not model 7's
     # freeing an evicted id drops it; its get is then NOT_FOUND
     assert s.free([4]) == OK and s.get_batch([4])[0] == NOT_FOUND
 
@@ -475,3 +481,106 @@ def test_pull_hand_trace():
     assert cons.pull(prod, [ib])[0] == NOSPACE and ib in prod.objects  # 3 + 3 pages > 4: nothing happens
     assert prod.objects[ib].consumers_left == 0
     assert cons.pull(OracleStore(4 * 128, 128), [1])[0] == INVALID        # page sizes differ
+
+
+def _mutant_most_recent_group_first(monkeypatch):
+    def victims(self, demand, pinned):
+        have = len(self.free_stack)
+        if have >= demand:
+            return []
+        cands = [o for o in self.objects if self.objects[o].evictable and self.objects[o].group not in pinned]
+        if have + sum(ostore.pages_for(self.objects[c].nbytes, self.page_bytes) for c in cands) < demand:
+            return None
+        cands.sort(key=lambda o: (-self.group_last[self.objects[o].group], -self.objects[o].order, -o))
+        out = []
+        for o in cands:
+            if have >= demand:
+                break
+            out.append(o)
+            have += ostore.pages_for(self.objects[o].nbytes, self.page_bytes)
+        return out
+    monkeypatch.setattr(OracleStore, "_victims", victims)
+
+
+def _mutant_ties_to_lowest_id(monkeypatch):
+    orig = OracleStore._victims
+
+    def victims(self, demand, pinned):
+        v = orig(self, demand, pinned)
+        if not v:
+            return v
+        cands = sorted((o for o in self.objects if self.objects[o].evictable and self.objects[o].group not in pinned),
+                       key=lambda o: (self.group_last[self.objects[o].group], -self.objects[o].order, o))
+        return cands[:len(v)]
+    monkeypatch.setattr(OracleStore, "_victims", victims)
+
+
+def _mutant_put_groups_not_pinned(monkeypatch):
+    orig = OracleStore._victims
+    monkeypatch.setattr(OracleStore, "_victims", lambda self, demand, pinned: orig(self, demand, set()))
+
+
+def _mutant_non_evictable_are_victims(monkeypatch):
+    orig = OracleStore._victims
+
+    def victims(self, demand, pinned):
+        flags = {o: self.objects[o].evictable for o in self.objects}
+        for o in self.objects.values():
+            o.evictable = True
+        try:
+            return orig(self, demand, pinned)
+        finally:
+            for o, f in flags.items():
+                if o in self.objects:
+                    self.objects[o].evictable = f
+    monkeypatch.setattr(OracleStore, "_victims", victims)
+
+
+def _mutant_nospace_evicts_anyway(monkeypatch):
+    orig = OracleStore.put_batch
+
+    def put_batch(self, items):
+        st, ids = orig(self, items)
+        if st == NOSPACE:
+            pinned = {int(it.group) for it in items}
+            for o in [o for o in self.objects if self.objects[o].evictable and self.objects[o].group not in pinned]:
+                self._release(o)
+                self.evicted.add(o)
+        return st, ids
+    monkeypatch.setattr(OracleStore, "put_batch", put_batch)
+
+
+def _mutant_get_does_not_touch(monkeypatch):
+    orig = OracleStore.get_batch
+
+    def get_batch(self, ids, casts=None):
+        saved = (self.clock, dict(self.group_last))
+        out = orig(self, ids, casts)
+        self.clock, self.group_last = saved[0], saved[1]
+        return out
+    monkeypatch.setattr(OracleStore, "get_batch", get_batch)
+
+
+def _mutant_evicts_whole_groups(monkeypatch):
+    orig = OracleStore._victims
+
+    def victims(self, demand, pinned):
+        v = orig(self, demand, pinned)
+        if not v:
+            return v
+        groups = {self.objects[o].group for o in v}
+        extra = sorted((o for o in self.objects if self.objects[o].evictable and self.objects[o].group in groups
+                        and o not in v), key=lambda o: (-self.objects[o].order, -o))
+        return v + extra
+    monkeypatch.setattr(OracleStore, "_victims", victims)
+
+
+@pytest.mark.parametrize("mutant", [_mutant_most_recent_group_first, _mutant_ties_to_lowest_id,
+                                    _mutant_put_groups_not_pinned, _mutant_non_evictable_are_victims,
+                                    _mutant_nospace_evicts_anyway, _mutant_get_does_not_touch,
+                                    _mutant_evicts_whole_groups])
+def test_planted_lru_mistakes_fail_the_hand_trace(monkeypatch, mutant):
+    """Each plausible misreading of the victim rule (reading 6; §5.3, "How
+    does it work?") planted in the oracle fails the hand-derived trace."""
+    mutant(monkeypatch)
+    assert _expect_failure(test_lru_reverse_layer_hand_trace)
