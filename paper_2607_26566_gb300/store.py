@@ -30,14 +30,20 @@ class T2IError(RuntimeError):
 
 
 def _ptr(x) -> int:
-    """Address of a tensor / array / int."""
+    """Address of a tensor / array / int. A buffer's bytes travel as one
+    range, so tensors and arrays must be contiguous (a strided view would
+    copy the wrong bytes, or overwrite its neighbours on a get)."""
     if x is None:
         return 0
     if isinstance(x, int):
         return x
     if hasattr(x, "data_ptr"):
+        if hasattr(x, "is_contiguous") and not x.is_contiguous():
+            raise ValueError("a tensor buffer must be contiguous (call .contiguous() first)")
         return int(x.data_ptr())
     if isinstance(x, np.ndarray):
+        if not x.flags.c_contiguous:
+            raise ValueError("an array buffer must be C-contiguous")
         return int(x.ctypes.data)
     raise TypeError(f"cannot take the address of {type(x)}")
 

@@ -76,3 +76,21 @@ def test_store_create_without_a_gpu_fails_cleanly(lib):
     st = lib.t2i_store_create(C.c_void_p(1 << 20), C.byref(cfg), 0, C.byref(h))
     assert st in (L.ERR_CUDA, L.ERR_INVALID) and not h.value
     assert lib.t2i_last_error(None)
+
+
+def test_strided_buffers_are_refused():
+    """A buffer travels as one byte range: strided tensors and arrays are
+    refused before any descriptor is built."""
+    import numpy as np
+    import torch
+
+    from paper_2607_26566_gb300 import get_descs, put_descs
+    t = torch.zeros(8, 6)
+    with pytest.raises(ValueError):
+        put_descs([t[:, :3]])
+    with pytest.raises(ValueError):
+        get_descs([1], [t.t()])
+    with pytest.raises(ValueError):
+        put_descs([np.zeros((4, 4), np.float32)[:, 1]])
+    d = put_descs([t[2:5], np.zeros(16, np.uint8)[4:]])   # contiguous slices are fine
+    assert list(d["nbytes"]) == [3 * 6 * 4, 12]
