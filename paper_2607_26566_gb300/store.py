@@ -206,7 +206,14 @@ class Ctl:
 
 class Store:
     """A store over a device pool (``t2i_store_create``). ``pool`` is a CUDA
-    tensor (kept alive by the store object) or an address with ``pool_bytes``."""
+    tensor (kept alive by the store object) or an address with ``pool_bytes``.
+
+    Calls are asynchronous like ``cudaMemcpyAsync``: a put source must keep
+    its bytes, and a get destination its memory, until the call's stream has
+    run the call. The binding does not hold the tensors named in descriptor
+    arrays. A tensor used on a stream other than the one it was allocated on
+    needs ``tensor.record_stream(stream)`` before it is dropped, as for any
+    cross-stream use under PyTorch's caching allocator."""
 
     def __init__(self, pool, page_bytes: int, pool_bytes: int | None = None, device: int | None = None,
                  h2d_mode: int = 0, check_pointers: int = 1, alloc_policy: int = 0):
