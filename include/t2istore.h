@@ -73,7 +73,13 @@ typedef struct t2i_store_config {
                                 1 = extent: the lowest run of enough consecutive free pages,
                                 else the lowest free pages (objects stay contiguous and can be
                                 used in place, see t2i_view)                                  */
-    uint32_t reserved;       /* must be 0                                                       */
+    uint32_t d2h_mode;       /* gets into pinned host memory: 0 = the get kernel writes host memory
+                                directly (zero-copy over the host link); 1 = items without the
+                                cast take one copy-engine cudaMemcpyAsync per run of consecutive
+                                pages, which leaves the SMs free for work in the other direction
+                                (a put from host on another stream); items with the cast always
+                                run in the kernel. Needs check_pointers = 1 (the store must see
+                                that a destination is host memory).                           */
 } t2i_store_config;
 
 /* ---- put ------------------------------------------------------------------
@@ -102,7 +108,8 @@ typedef struct t2i_put_desc {
  * produced tensor into its own memory), optionally casting fp32 -> bf16.  */
 typedef struct t2i_get_desc {
     t2i_id id;
-    void* dst;            /* device memory of the store's device, or pinned host memory      */
+    void* dst;            /* device memory of the store's device, or pinned host memory (written
+                             by the kernel, or by the copy engine under d2h_mode = 1)         */
     uint64_t dst_bytes;   /* capacity at dst: >= nbytes, or >= nbytes / 2 with cast = 1       */
     uint32_t cast;        /* 0 = bytes as stored; 1 = the object is little-endian fp32 and dst
                              receives bf16, round to nearest even (NaN -> quiet NaN with the
@@ -127,6 +134,7 @@ typedef struct t2i_stats {
     uint64_t h2d_copies; /* copy-engine copies issued for host sources                        */
     uint64_t reclaimed;  /* objects freed by the store after their last declared consumer    */
     uint64_t views;      /* successful t2i_view calls                                         */
+    uint64_t d2h_copies; /* copy-engine copies issued for host destinations (d2h_mode = 1)       */
 } t2i_stats;
 
 typedef struct t2i_object_info {
@@ -173,7 +181,10 @@ t2i_status t2i_put_batch(t2i_store* store, const t2i_put_desc* descs, uint32_t n
                          void* cuda_stream);
 
 /* Copies n objects into their destinations (paper §5.2 "consumer pulls").
- * Every item is validated first; per_item (nullable, n entries) receives
+ * The copies are one kernel launch per batch (more only when the
+ * descriptors exceed one launch's parameter space), plus, under d2h_mode =
+ * 1, one copy-engine copy per run of consecutive pages of each item without
+ * the cast whose destination is pinned host memory. Every item is validated first; per_item (nullable, n entries) receives
  * OK / NOT_FOUND / EVICTED / INVALID per item. If any item fails, the call
  * returns the first failing status in descriptor order and writes nothing.
  * The same id may appear more than once. Objects reserved with src = NULL

@@ -17,7 +17,7 @@ STATUS_NAMES = {0: "OK", 1: "INVALID", 2: "NOSPACE", 3: "NOT_FOUND", 4: "EVICTED
 
 class StoreConfig(C.Structure):
     _fields_ = [("pool_bytes", C.c_uint64), ("page_bytes", C.c_uint64), ("h2d_mode", C.c_uint32),
-                ("check_pointers", C.c_uint32), ("alloc_policy", C.c_uint32), ("reserved", C.c_uint32)]
+                ("check_pointers", C.c_uint32), ("alloc_policy", C.c_uint32), ("d2h_mode", C.c_uint32)]
 
 
 class PutDesc(C.Structure):
@@ -39,7 +39,7 @@ class Stats(C.Structure):
     _fields_ = [(n, C.c_uint64) for n in (
         "total_pages", "limit_pages", "used_pages", "free_pages", "live_objects",
         "bytes_put", "bytes_got", "puts", "gets", "misses", "evictions",
-        "pages_moved", "bytes_moved", "launches", "h2d_copies", "reclaimed", "views")]
+        "pages_moved", "bytes_moved", "launches", "h2d_copies", "reclaimed", "views", "d2h_copies")]
 
     def as_dict(self) -> dict:
         return {n: int(getattr(self, n)) for n, _ in self._fields_}

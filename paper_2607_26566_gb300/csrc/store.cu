@@ -305,7 +305,7 @@ t2i_status Store::check_user(const void* p, uint64_t n, bool want_write, bool is
                 return T2I_ERR_INVALID;
             }
             *dev_addr = r.dev_base + (a - r.start);
-            *needs_copy_engine = !want_write && cfg_.h2d_mode == 1;
+            *needs_copy_engine = want_write ? cfg_.d2h_mode == 1 : cfg_.h2d_mode == 1;
             break;
         case MemKind::Unknown:
             // pageable host memory: only a host source, through the copy engine
@@ -441,6 +441,7 @@ t2i_status Store::get(const t2i_get_desc* descs, uint32_t n, t2i_status* per_ite
     // 1. directory (ids, evictions, cast rules) without touching the LRU
     std::vector<t2i_status> per(n, T2I_OK);
     std::vector<uint64_t> dev_dst(n, 0);
+    std::vector<uint8_t> use_ce(n, 0);
     t2i_status first = T2I_OK;
     uint32_t first_i = 0;
     Range cache;
@@ -460,6 +461,7 @@ t2i_status Store::get(const t2i_get_desc* descs, uint32_t n, t2i_status* per_ite
             } else {
                 bool ce = false;
                 if (check_user(d.dst, out_bytes, true, false, &dev_dst[i], &ce, &cache) != T2I_OK) s = T2I_ERR_INVALID;
+                use_ce[i] = ce && !d.cast;  // the cast runs in the kernel
             }
         }
         per[i] = s;
@@ -492,23 +494,50 @@ t2i_status Store::get(const t2i_get_desc* descs, uint32_t n, t2i_status* per_ite
     }
     segs_.clear();
     deps_.begin(si);
+    bool any = false;
     for (uint32_t i = 0; i < n; ++i) {
         const Object* o = objs_[i];
         if (o->nbytes == 0) continue;
         for (uint32_t pg : o->pages) deps_.reads(pg);
+        any = true;
+        if (use_ce[i]) continue;
         segs_.push_back({dev_dst[i], o->nbytes | (descs[i].cast ? kCastFlag : 0), o->pages.data(),
                          uint32_t(o->pages.size())});
     }
-    if (!segs_.empty()) {
+    if (any) {
         cudaError_t we = deps_.wait();
         if (we != cudaSuccess) return cuda_fail("get: cannot order after earlier calls", we);
-        st = launch_segments<Mode::Get>(segs_, stream);
-        // the pages carry this call as a reader even when it failed part-way
-        // (launches before the failure may still be reading them)
+        st = segs_.empty() ? T2I_OK : launch_segments<Mode::Get>(segs_, stream);
+        // items for the copy engine (pinned host destinations, d2h_mode = 1):
+        // one copy per run of consecutive pages
+        const uint64_t P = uint64_t(1) << page_shift_;
+        for (uint32_t i = 0; i < n && st == T2I_OK; ++i) {
+            const Object* o = objs_[i];
+            if (!use_ce[i] || o->nbytes == 0) continue;
+            char* dst = static_cast<char*>(descs[i].dst);
+            size_t j = 0;
+            while (j < o->pages.size()) {
+                size_t k = j + 1;
+                while (k < o->pages.size() && o->pages[k] == o->pages[k - 1] + 1) ++k;
+                const uint64_t off = j * P;
+                const uint64_t bytes = std::min<uint64_t>(o->nbytes - off, (k - j) * P);
+                cudaError_t e = cudaMemcpyAsync(dst + off, reinterpret_cast<const void*>(pool_ + uint64_t(o->pages[j]) * P),
+                                                bytes, cudaMemcpyDeviceToHost, stream);
+                if (e != cudaSuccess) {
+                    st = cuda_fail("get: host copy failed", e);
+                    break;
+                }
+                ctl_.counters().d2h_copies++;
+                j = k;
+            }
+        }
+        // every page of the batch carries this call as a reader, even when it
+        // failed part-way (copies enqueued before the failure may still be
+        // reading them)
         uint32_t q = 0;
         cudaError_t ee = deps_.end(&q);
-        for (const Seg& sg : segs_)
-            for (uint32_t k = 0; k < sg.n_pages; ++k) deps_.mark_read(sg.pages[k], q);
+        for (uint32_t i = 0; i < n; ++i)
+            for (uint32_t pg : objs_[i]->pages) deps_.mark_read(pg, q);
         if (st != T2I_OK) return st;  // nothing was counted: the get did not happen
         if (ee != cudaSuccess) st = cuda_fail("get: cannot record its event", ee);
     }
@@ -812,7 +841,7 @@ t2i_status t2i_store_create(void* pool_dev, const t2i_store_config* cfg, int dev
         return T2I_ERR_INVALID;
     }
     if (cfg->pool_bytes / cfg->page_bytes > 0xFFFFFFFFull || cfg->h2d_mode > 1 || cfg->check_pointers > 1 ||
-        cfg->alloc_policy > 1 || cfg->reserved != 0) {
+        cfg->alloc_policy > 1 || cfg->d2h_mode > 1) {
         t2i::set_thread_error("t2i_store_create: too many pages or a bad flag");
         return T2I_ERR_INVALID;
     }

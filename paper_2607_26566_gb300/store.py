@@ -216,7 +216,7 @@ class Store:
     cross-stream use under PyTorch's caching allocator."""
 
     def __init__(self, pool, page_bytes: int, pool_bytes: int | None = None, device: int | None = None,
-                 h2d_mode: int = 0, check_pointers: int = 1, alloc_policy: int = 0):
+                 h2d_mode: int = 0, check_pointers: int = 1, alloc_policy: int = 0, d2h_mode: int = 0):
         self._lib = L.load()
         self.pool = pool
         if pool_bytes is None:
@@ -226,7 +226,7 @@ class Store:
         self.device = device
         self.page_bytes = int(page_bytes)
         self.pool_bytes = int(pool_bytes)
-        cfg = L.StoreConfig(pool_bytes, page_bytes, h2d_mode, check_pointers, alloc_policy, 0)
+        cfg = L.StoreConfig(pool_bytes, page_bytes, h2d_mode, check_pointers, alloc_policy, d2h_mode)
         h = C.c_void_p()
         st = self._lib.t2i_store_create(C.c_void_p(_ptr(pool)), C.byref(cfg), device, C.byref(h))
         if st != L.OK:

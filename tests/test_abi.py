@@ -94,3 +94,15 @@ def test_strided_buffers_are_refused():
         put_descs([np.zeros((4, 4), np.float32)[:, 1]])
     d = put_descs([t[2:5], np.zeros(16, np.uint8)[4:]])   # contiguous slices are fine
     assert list(d["nbytes"]) == [3 * 6 * 4, 12]
+
+
+def test_store_create_refuses_bad_flags(lib):
+    """Flags are checked before the device is touched (no GPU needed)."""
+    for fields in ({"d2h_mode": 2}, {"h2d_mode": 2}, {"alloc_policy": 2}, {"check_pointers": 2}):
+        cfg = L.StoreConfig(1 << 20, 1 << 16, 0, 1, 0, 0)
+        for k, v in fields.items():
+            setattr(cfg, k, v)
+        h = C.c_void_p()
+        st = lib.t2i_store_create(C.c_void_p(1 << 21), C.byref(cfg), 0, C.byref(h))
+        assert st == L.ERR_INVALID and not h.value, fields
+        assert b"bad flag" in lib.t2i_last_error(None)

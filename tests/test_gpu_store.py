@@ -279,6 +279,79 @@ def test_host_sources_and_destinations(h2d_mode):
     assert stats["launches"] >= (2 if h2d_mode == 0 else 1)
 
 
+@pytest.mark.parametrize("h2d_mode", [0, 1])
+def test_copy_engine_gets_into_host(h2d_mode):
+    """d2h_mode = 1: gets into pinned host memory take the copy engine (one
+    copy per run of consecutive pages, any alignment), items with the cast
+    and device destinations stay in the kernel, all in one call."""
+    rng = np.random.default_rng(11)
+    P = 64 * 1024
+    st = make_store(256 * P, P, h2d_mode=h2d_mode, d2h_mode=1)
+    ora = OracleStore(256 * P, P)
+    # fragment the free stack so that page lists break into several runs
+    s, filler = st.put_batch(put_descs([0] * 6, nbytes=[7 * P] * 6))
+    assert s == 0 and st.free([int(x) for x in filler[::2]]) == 0
+    ora.put_batch([PutItem(7 * P) for _ in range(6)])
+    ora.free([1, 3, 5])
+    sizes = (1, 100, P, 3 * P + 17, 9 * P + 5, 12345)
+    datas = [rng.integers(0, 256, n, dtype=np.uint8) for n in sizes]
+    f = rng.standard_normal(3 * P // 4 + 3).astype(np.float32)
+    f[:4] = [np.inf, -np.inf, np.nan, -0.0]
+    datas.append(f.view(np.uint8))
+    srcs = [torch.from_numpy(d).to(DEV) for d in datas]
+    s, ids = st.put_batch(put_descs(srcs))
+    assert s == 0, st.last_error()
+    _, oids = ora.put_batch([PutItem(d.size, d) for d in datas])
+    assert [int(i) for i in ids] == oids
+    compare_meta(st, ora)
+    big = torch.zeros(sum(sizes) + 64, dtype=torch.uint8).pin_memory()
+    offs = np.cumsum([3] + [n + 5 for n in sizes[:-1]])           # odd offsets: unaligned host pointers
+    host_outs = [big[int(o):int(o) + n] for o, n in zip(offs, sizes)]
+    cast_out = torch.empty(f.size, dtype=torch.bfloat16).pin_memory()
+    dev_out = torch.empty(sizes[3], dtype=torch.uint8, device=DEV)
+    gd = get_descs([int(i) for i in ids[:6]] + [int(ids[6]), int(ids[3])], host_outs + [cast_out, dev_out],
+                   cast=[0] * 6 + [1, 0])
+    launches0, d2h0 = st.stats()["launches"], st.stats()["d2h_copies"]
+    s, per = st.get_batch(gd)
+    assert s == 0 and list(per) == [0] * 8, st.last_error()
+    torch.cuda.synchronize()
+    for o, d in zip(host_outs, datas):
+        assert np.array_equal(o.numpy(), d)
+    assert np.array_equal(cast_out.view(torch.int16).numpy().view(np.uint16),
+                          f32_bits_to_bf16_bits(f.view(np.uint32)))
+    assert np.array_equal(dev_out.cpu().numpy(), datas[3])
+    stats = st.stats()
+    assert stats["launches"] - launches0 == 1          # the cast and the device destination
+    runs = sum(1 + sum(1 for a, b in zip(ps, ps[1:]) if b != a + 1)
+               for ps in (ora.pages_of(i) for i in oids[:6]))
+    assert stats["d2h_copies"] - d2h0 == runs and runs > 6
+
+
+def test_copy_engine_get_orders_before_page_reuse():
+    """A copy-engine get on one stream, then a put on another stream that
+    reuses the pages: the put waits for the copy (write after read)."""
+    P = 2 << 20
+    st = make_store(64 * P, P, d2h_mode=1)
+    s1, s2, s3 = torch.cuda.Stream(), torch.cuda.Stream(), torch.cuda.Stream()
+    a = torch.randint(0, 256, (64 * P,), dtype=torch.uint8, device=DEV)
+    b = torch.randint(0, 256, (64 * P,), dtype=torch.uint8, device=DEV)
+    host = torch.empty(64 * P, dtype=torch.uint8).pin_memory()
+    want = a.cpu()
+    torch.cuda.synchronize()
+    for _ in range(3):
+        s, (i,) = st.put_batch(put_descs([a]), stream=s1)
+        assert s == 0
+        s, _ = st.get_batch(get_descs([int(i)], [host]), stream=s2)
+        assert s == 0
+        assert st.free([int(i)]) == 0
+        s, (j,) = st.put_batch(put_descs([b]), stream=s3)     # the same pages
+        assert s == 0
+        torch.cuda.synchronize()
+        assert torch.equal(host, want)
+        assert st.free([int(j)]) == 0
+    assert st.stats()["d2h_copies"] >= 3
+
+
 def test_streams_are_ordered():
     """Put on one stream, get on another, free, re-put on a third: the store
     orders its own work across streams."""
