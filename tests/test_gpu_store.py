@@ -325,6 +325,11 @@ def test_copy_engine_gets_into_host(h2d_mode):
     runs = sum(1 + sum(1 for a, b in zip(ps, ps[1:]) if b != a + 1)
                for ps in (ora.pages_of(i) for i in oids[:6]))
     assert stats["d2h_copies"] - d2h0 == runs and runs > 6
+    # pageable destinations stay refused: nothing is enqueued or written
+    pageable = np.full(sizes[2], 7, np.uint8)
+    s, per = st.get_batch(get_descs([int(ids[2])], [pageable]))
+    assert s == 1 and list(per) == [1] and (pageable == 7).all()
+    assert st.stats()["d2h_copies"] == stats["d2h_copies"]
 
 
 def test_copy_engine_get_orders_before_page_reuse():
