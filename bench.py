@@ -1609,6 +1609,17 @@ def oracle_row_samples(rows: dict) -> None:
 
 
 # ----------------------------------------------------------------------------- main
+def arm_config(args, world: int) -> dict:
+    """The workload both arms name (the reference arm times a bounded sample
+    of it, described in its ``cpu_baseline.sample``)."""
+    pool_bytes = int(args.pool_gib * (1 << 30)) if args.pool_gib else None
+    return {"workload": f"t2i handoff, B={args.batch}, {args.requests} requests in flight",
+            "streams": args.streams,
+            "pool_bytes": pool_bytes or W.HANDOFF["pool_bytes"], "page_bytes": W.HANDOFF["page_bytes"],
+            "bytes_per_step": hw_bytes(args.batch, args.requests), "l2": "inputs > L2 (no flush)",
+            "parallelism": f"replicas x{world}"}
+
+
 def run_reference(args, dist_ctx):
     if dist_ctx.rank != 0:
         return
@@ -1618,6 +1629,7 @@ def run_reference(args, dist_ctx):
         oracle_sample(B, 1)
     vals = []
     t0 = time.perf_counter()
+    nb = 0
     for _ in range(args.steps):
         v, dt, nb, _ = oracle_sample(B, n_req)
         vals.append((v, dt))
@@ -1629,11 +1641,12 @@ def run_reference(args, dist_ctx):
         "impl": "reference", "metric": METRIC, "value": round(value, 3), "unit": "GB/s", "n_gpus": args.gpus,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms, 3), "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "u8+f32->bf16", "data": "synthetic",
-        "config": {"workload": f"t2i handoff, B={B}, {n_req} requests per step (bounded sample of 64)",
-                   "pool_bytes": W.HANDOFF["pool_bytes"], "page_bytes": W.HANDOFF["page_bytes"]},
+        "config": arm_config(args, dist_ctx.world),
         "cpu_baseline": {"value": round(value, 3), "unit": "GB/s", "cores": 1, "kind": "oracle",
-                         "sample": f"{n_req} of 64 requests per step, numpy oracle, single thread"},
+                         "sample": f"each step: {n_req} of the step's {args.requests} B={B} requests (put, get with "
+                                   f"the latents cast, free), numpy oracle, single thread"},
         "e2e": {"value": round(value, 3), "unit": "GB/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+        "sampled_bytes_per_step": int(nb),   # ms_per_step is the time of this sample
         "wall_s": round(time.perf_counter() - t0, 2),
     }
     print(json.dumps(line), flush=True)
@@ -1842,11 +1855,7 @@ def main():
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms_max / args.steps, 4),
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "u8+f32->bf16",
             "data": "synthetic",
-            "config": {"workload": f"t2i handoff, B={B}, {args.requests} requests in flight",
-                       "streams": args.streams,
-                       "pool_bytes": pool_bytes or W.HANDOFF["pool_bytes"], "page_bytes": W.HANDOFF["page_bytes"],
-                       "bytes_per_step": hw_bytes(B, args.requests), "l2": "inputs > L2 (no flush)",
-                       "parallelism": f"replicas x{dist_ctx.world}"},
+            "config": arm_config(args, dist_ctx.world),
             "hbm_frac": round(value / dist_ctx.world / peak, 4), "hbm_frac_nominal_8tbs": round(value / dist_ctx.world / 8000.0, 4),
             "step_ms": kern["step_ms"], "per_call": per_call,
             "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e, "gpu_launches": int(launches),
