@@ -288,9 +288,10 @@ const t2i_ctl* t2i_store_ctl(const t2i_store* store);
 
 /* Message of the last failed call on this store (or, for NULL, of the last
  * failed call on this thread that has no store: t2i_store_create,
- * t2i_ctl_create, t2i_gather_noalloc, the prefix calls). Never NULL. A store's message lives inside the store: it stays
- * valid until the next call on that store, from any thread, or its
- * destruction; copy it out before then.                                    */
+ * t2i_ctl_create, t2i_gather_noalloc, the prefix calls). Never NULL. A
+ * store's message lives inside the store: it stays valid until the next
+ * call on that store, from any thread, or its destruction; copy it out
+ * before then.                                                              */
 const char* t2i_last_error(const t2i_store* store);
 
 /* =========================================================================

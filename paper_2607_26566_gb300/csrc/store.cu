@@ -521,8 +521,8 @@ t2i_status Store::get(const t2i_get_desc* descs, uint32_t n, t2i_status* per_ite
                 while (k < o->pages.size() && o->pages[k] == o->pages[k - 1] + 1) ++k;
                 const uint64_t off = j * P;
                 const uint64_t bytes = std::min<uint64_t>(o->nbytes - off, (k - j) * P);
-                cudaError_t e = cudaMemcpyAsync(dst + off, reinterpret_cast<const void*>(pool_ + uint64_t(o->pages[j]) * P),
-                                                bytes, cudaMemcpyDeviceToHost, stream);
+                const void* src = reinterpret_cast<const void*>(pool_ + uint64_t(o->pages[j]) * P);
+                cudaError_t e = cudaMemcpyAsync(dst + off, src, bytes, cudaMemcpyDeviceToHost, stream);
                 if (e != cudaSuccess) {
                     st = cuda_fail("get: host copy failed", e);
                     break;

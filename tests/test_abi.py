@@ -106,3 +106,105 @@ def test_store_create_refuses_bad_flags(lib):
         st = lib.t2i_store_create(C.c_void_p(1 << 21), C.byref(cfg), 0, C.byref(h))
         assert st == L.ERR_INVALID and not h.value, fields
         assert b"bad flag" in lib.t2i_last_error(None)
+
+
+C_DRIVER = r"""
+#include <stdio.h>
+#include <string.h>
+#include "t2istore.h"
+
+static t2i_put_desc pd(uint64_t nbytes, uint64_t group, uint32_t order, uint32_t evictable) {
+    t2i_put_desc d;
+    memset(&d, 0, sizeof d);
+    d.nbytes = nbytes;
+    d.group = group;
+    d.order = order;
+    d.evictable = evictable;
+    return d;
+}
+static void show_pages(const t2i_ctl* c, t2i_id id) {
+    t2i_object_info info;
+    uint32_t pg[16];
+    t2i_ctl_object(c, id, &info, pg, 16);
+    printf("pages %llu:", (unsigned long long)id);
+    for (uint32_t i = 0; i < info.n_pages; ++i) printf(" %u", pg[i]);
+    printf("\n");
+}
+static void show_evictions(const t2i_ctl* c) {
+    t2i_id ev[16];
+    uint64_t n = 0;
+    t2i_ctl_last_evictions(c, ev, 16, &n);
+    printf("evicted:");
+    for (uint64_t i = 0; i < n; ++i) printf(" %llu", (unsigned long long)ev[i]);
+    printf("\n");
+}
+int main(void) {
+    const uint64_t P = 1024;
+    t2i_ctl* c = NULL;
+    if (t2i_ctl_create(6, P, 0, &c) != T2I_OK) return 1;
+    t2i_put_desc w1[3] = {pd(P, 1, 0, 1), pd(P, 1, 1, 1), pd(P, 1, 2, 1)};
+    t2i_put_desc w2[2] = {pd(P, 2, 0, 1), pd(P, 2, 1, 1)};
+    t2i_id ids[4];
+    printf("put %d\n", t2i_ctl_put(c, w1, 3, ids));
+    printf("put %d\n", t2i_ctl_put(c, w2, 2, ids));
+    t2i_get_desc g;
+    memset(&g, 0, sizeof g);
+    g.id = 1;
+    printf("get %d\n", t2i_ctl_get(c, &g, 1, NULL));
+    t2i_put_desc x = pd(3 * P, 3, 0, 0);
+    printf("put %d\n", t2i_ctl_put(c, &x, 1, ids));
+    show_evictions(c);
+    show_pages(c, ids[0]);
+    t2i_get_desc g3[3];
+    memset(g3, 0, sizeof g3);
+    g3[0].id = 4;
+    g3[1].id = 99;
+    g3[2].id = 1;
+    t2i_status per[3];
+    const t2i_status gs = t2i_ctl_get(c, g3, 3, per);
+    printf("get %d per %d %d %d\n", gs, per[0], per[1], per[2]);
+    t2i_put_desc y = pd(P, 2, 0, 1);
+    printf("put %d\n", t2i_ctl_put(c, &y, 1, ids));
+    show_evictions(c);
+    show_pages(c, ids[0]);
+    t2i_put_desc big = pd(4 * P, 4, 0, 0);
+    printf("put %d\n", t2i_ctl_put(c, &big, 1, ids));
+    show_evictions(c);
+    t2i_stats s;
+    t2i_ctl_stats(c, &s);
+    printf("used %llu free %llu evictions %llu\n", (unsigned long long)s.used_pages, (unsigned long long)s.free_pages,
+           (unsigned long long)s.evictions);
+    t2i_ctl_destroy(c);
+    return 0;
+}
+"""
+
+C_DRIVER_WANT = """put 0
+put 0
+get 0
+put 0
+evicted: 5 4
+pages 6: 3 4 5
+get 4 per 4 3 0
+put 0
+evicted: 3
+pages 7: 2
+put 2
+evicted:
+used 6 free 0 evictions 3
+"""
+
+
+def test_control_core_from_c_follows_the_hand_trace(lib, tmp_path):
+    """A plain C program linked against the library drives the host control
+    core through the C ABI: the LRU victims and pages worked out by hand from
+    §5.3 and the readings of the LRU and placement rules (the same trace the
+    oracle is pinned by)."""
+    src = tmp_path / "drive.c"
+    src.write_text(C_DRIVER)
+    exe = tmp_path / "drive"
+    lib_dir = os.path.dirname(L.LIB_PATH)
+    subprocess.run(["gcc", "-std=c99", "-Wall", "-Werror", "-I" + os.path.join(ROOT, "include"), str(src), "-o",
+                    str(exe), "-L" + lib_dir, "-l:libt2istore.so", "-Wl,-rpath," + lib_dir], check=True)
+    out = subprocess.run([str(exe)], capture_output=True, text=True, check=True).stdout
+    assert out == C_DRIVER_WANT
