@@ -1799,7 +1799,7 @@ def main():
     e2e = None
     if not args.no_e2e:
         he = Handoff(B, args.requests, device, host_buffers=True)
-        e_steps = max(2, min(args.steps, 3))
+        e_steps = max(2, min(args.steps, 10))
         # the kernels read and write host memory themselves (h2d_mode = d2h_mode = 0)
         ms_e, _, _, _ = time_handoff(he, e_steps, 3, dist_ctx, per_kernel=False, n_streams=args.streams,
                                      nvtx="bench_e2e")
