@@ -59,7 +59,7 @@ def parse():
     p.add_argument("--no-sweep", action="store_true", help="skip timing B = 1 and B = 4")
     p.add_argument("--pool-gib", type=float, default=None, help="smaller pool (profiling small cases)")
     p.add_argument("--cpu-seconds", type=float, default=10.0, help="minimum CPU-baseline sample time")
-    p.add_argument("--rows", default="tiny,weights,adapters,compaction,prefix,views,pull",
+    p.add_argument("--rows", default="tiny,weights,adapters,compaction,prefix,views,pull,host",
                    help="other hot-path rows timed in the same run (comma list, or 'none')")
     p.add_argument("--adapter-calls", type=int, default=10_000)
     p.add_argument("--adapter-sets", type=int, default=None, help="fewer LoRA sets (profiling small cases)")
@@ -1608,6 +1608,101 @@ def oracle_row_samples(rows: dict) -> None:
                                                  f"compact of a 4 GiB paged pool to 3/4 ({len(moves)} pages moved)")
 
 
+# ----------------------------------------------------------------------------- host control
+def time_host_control(reps: int = 200) -> dict:
+    """The host steps of the path (§8 a1, a2, a7, a9) alone, through the
+    store's control core (t2i_ctl_*: the same code every store runs before
+    its launches), on the host: median µs per call."""
+    from paper_2607_26566_gb300 import Ctl, get_descs, put_descs
+
+    def med(fn, n):
+        ts = []
+        for _ in range(n):
+            t = time.perf_counter()
+            fn()
+            ts.append(time.perf_counter() - t)
+        return round(1e6 * statistics.median(ts), 2)
+
+    out = {"workload": "host control core alone (t2i_ctl_*), median µs per call"}
+    # a1 + a2 + a9: put and free of one B=8 handoff request (4 objects, 45 pages of 2 MiB)
+    C_ = W.HANDOFF
+    specs = W.handoff_specs(8)
+    ctl = Ctl(C_["pool_bytes"] // C_["page_bytes"], C_["page_bytes"])
+    pd = put_descs([0] * len(specs), nbytes=[sp.nbytes for sp in specs])
+    ids = [None]
+
+    def put():
+        st, ids[0] = ctl.put(pd)
+        assert st == 0
+
+    def free():
+        assert ctl.free(ids[0]) == 0
+
+    put_t, free_t = [], []
+    for _ in range(reps):
+        t = time.perf_counter()
+        put()
+        put_t.append(time.perf_counter() - t)
+        t = time.perf_counter()
+        free()
+        free_t.append(time.perf_counter() - t)
+    out["handoff_put_us"] = round(1e6 * statistics.median(put_t), 2)
+    out["handoff_free_us"] = round(1e6 * statistics.median(free_t), 2)
+    put()
+    gd = get_descs(ids[0])
+    out["handoff_get_us"] = med(lambda: ctl.get(gd), reps)
+    ctl.close()
+    # a7: adapter sets (836 objects each, 256 KiB pages, 16 GiB pool); once
+    # the pool is full every set put evicts the least recently used set
+    A = W.ADAPTERS
+    ctl = Ctl(A["pool_bytes"] // A["page_bytes"], A["page_bytes"])
+    ranks = W.lora_ranks(0)
+    sets = []
+    for s_, r in enumerate(ranks[:64]):
+        objs = W.lora_objects(int(r))
+        sets.append(put_descs([0] * len(objs), nbytes=[nb for _, nb in objs], group=s_,
+                              order=[b for b, _ in objs], evictable=1))
+    put_t, evicted, live = [], 0, {}
+    for k in range(3 * len(sets)):
+        s_ = k % len(sets)
+        t = time.perf_counter()
+        st, got = ctl.put(sets[s_])
+        put_t.append(time.perf_counter() - t)
+        assert st == 0
+        ev = ctl.last_evictions()
+        evicted += len(ev)
+        live[s_] = got
+    steady = put_t[len(sets):]
+    out["adapter_set_put_us"] = round(1e6 * statistics.median(steady), 2)
+    out["adapter_set_put_evictions_per_call"] = round(evicted / len(put_t), 1)
+    # the 256-object hit get of one resident window (validation + LRU stamps)
+    last = (3 * len(sets) - 1) % len(sets)
+    gd = get_descs(live[last][:256])
+    out["adapter_get_256_us"] = med(lambda: ctl.get(gd), reps)
+    ctl.close()
+    # a8: compaction planning of the 64 GiB, 100,000-op fragmentation trace
+    C5 = W.COMPACTION
+    P = C5["page_bytes"]
+    tr = W.compaction_trace(1, C5["pool_bytes"] // P, P, C5["n_ops"], C5["lo"], C5["hi"], C5["p_free"],
+                            C5["settle_frac"])
+    ctl = Ctl(C5["pool_bytes"] // P, P)
+    oid = {}
+    for op in tr.ops:
+        if op[0] == "alloc":
+            st, got = ctl.put(put_descs([0], nbytes=[op[2]]))
+            assert st == 0
+            oid[op[1]] = int(got[0])
+        else:
+            assert ctl.free([oid.pop(op[1])]) == 0
+    t = time.perf_counter()
+    st, moves = ctl.compact(C5["limit_bytes"])
+    out["compaction_plan_ms"] = round(1e3 * (time.perf_counter() - t), 3)
+    out["compaction_moves"] = int(len(moves)) if st == 0 else None
+    ctl.close()
+    out["note"] = "through the Python binding (ctypes, descriptor arrays built beforehand)"
+    return out
+
+
 # ----------------------------------------------------------------------------- main
 def arm_config(args, world: int) -> dict:
     """The workload both arms name (the reference arm times a bounded sample
@@ -1657,6 +1752,8 @@ def run_rows(args, device, peak):
     wanted = [] if args.rows == "none" else [r.strip() for r in args.rows.split(",") if r.strip()]
     if "tiny" in wanted:
         rows["tiny"] = time_tiny(device)
+    if "host" in wanted:
+        rows["host"] = time_host_control()
     if "weights" in wanted:
         rows["weights"] = time_weights(device, n_blocks=args.weight_blocks)
     if "adapters" in wanted:
