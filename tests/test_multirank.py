@@ -87,3 +87,31 @@ def test_reference_arm_line_has_the_contract_keys():
     assert {"value", "unit", "cores", "kind", "sample"} <= set(d["cpu_baseline"])
     assert d["e2e"]["h2d_bytes_per_step"] == 0 and d["e2e"]["d2h_bytes_per_step"] == 0
     assert "workload" in d["config"]
+
+
+def test_host_row_plans_the_oracle_compaction(lib):
+    """bench.py's rows.host (the host steps through the control core, no
+    GPU): every figure is present and positive, and its compaction plan of
+    the 64 GiB fragmentation trace moves exactly the oracle's pages."""
+    import bench
+    import workloads as W
+    from oracle import OracleStore, PutItem
+
+    h = bench.time_host_control(reps=5)
+    for k in ("handoff_put_us", "handoff_free_us", "handoff_get_us", "adapter_set_put_us", "adapter_get_256_us",
+              "compaction_plan_ms"):
+        assert h[k] > 0, k
+    assert h["adapter_set_put_evictions_per_call"] > 0
+    C5 = W.COMPACTION
+    P = C5["page_bytes"]
+    tr = W.compaction_trace(1, C5["pool_bytes"] // P, P, C5["n_ops"], C5["lo"], C5["hi"], C5["p_free"],
+                            C5["settle_frac"])
+    ora = OracleStore(C5["pool_bytes"], P, keep_bytes=False)
+    ids = {}
+    for op in tr.ops:
+        if op[0] == "alloc":
+            ids[op[1]] = ora.put_batch([PutItem(op[2])])[1][0]
+        else:
+            ora.free([ids.pop(op[1])])
+    st, moves = ora.compact(C5["limit_bytes"])
+    assert st == 0 and h["compaction_moves"] == len(moves)
