@@ -353,15 +353,67 @@ __device__ __forceinline__ void cta_cast_aligned(unsigned char* __restrict__ dst
     }
 }
 
-// Same cast into a destination that is only 2-byte aligned: one element per
-// thread step.
-__device__ __forceinline__ void cta_cast_scalar(unsigned char* __restrict__ dst, const unsigned char* __restrict__ src,
-                                                uint32_t len) {
+// Blocks of 8 floats whose words start Q (0..3) words past the aligned
+// vectors a[2v]: each is cut out of a[2v], a[2v+1] and (Q > 0) a[2v+2],
+// cast, and stored as one 16-byte vector d[v]. Every aligned load holds at
+// least one word of the block, so no access leaves the source allocation.
+template <int Q, int S>
+__device__ __forceinline__ void cast_blocks_shifted(uint4* __restrict__ d, const uint4* __restrict__ a, uint32_t n8) {
+#pragma unroll 1
+    for (uint32_t base = 0; base < n8; base += kThreads * S) {
+        uint4 x[S], y[S], z[S];
+#pragma unroll
+        for (int j = 0; j < S; ++j) {
+            const uint32_t v = base + j * kThreads + threadIdx.x;
+            if (v < n8) {
+                x[j] = ld_stream(a + 2 * v);
+                y[j] = ld_stream(a + 2 * v + 1);
+                if (Q > 0) z[j] = ld_stream(a + 2 * v + 2);
+            }
+        }
+#pragma unroll
+        for (int j = 0; j < S; ++j) {
+            const uint32_t v = base + j * kThreads + threadIdx.x;
+            if (v < n8) {
+                const uint32_t w[12] = {x[j].x, x[j].y, x[j].z, x[j].w, y[j].x, y[j].y,
+                                        y[j].z, y[j].w, Q > 0 ? z[j].x : 0u, Q > 0 ? z[j].y : 0u,
+                                        Q > 0 ? z[j].z : 0u, 0u};
+                uint4 o;
+                o.x = pack_bf16x2(w[Q + 0], w[Q + 1]);
+                o.y = pack_bf16x2(w[Q + 2], w[Q + 3]);
+                o.z = pack_bf16x2(w[Q + 4], w[Q + 5]);
+                o.w = pack_bf16x2(w[Q + 6], w[Q + 7]);
+                st_stream(d + v, o);
+            }
+        }
+    }
+}
+
+// Same cast into a destination that is only 2-byte aligned. The first
+// h < 8 elements, one per thread, bring the destination to a 16-byte
+// boundary; the source (16-byte aligned) is then h words past one, so the
+// blocks of 8 are cut out of aligned loads (cast_blocks_shifted); the last
+// < 8 elements one per thread.
+__device__ __forceinline__ void cta_cast_any(unsigned char* __restrict__ dst, const unsigned char* __restrict__ src,
+                                             uint32_t len) {
     const uint32_t nf = len >> 2;
     const uint32_t* s = reinterpret_cast<const uint32_t*>(src);
-    uint16_t* d = reinterpret_cast<uint16_t*>(dst);
-#pragma unroll 1
-    for (uint32_t i = threadIdx.x; i < nf; i += kThreads) d[i] = (uint16_t)bf16_rne_bits(s[i]);
+    uint16_t* d16 = reinterpret_cast<uint16_t*>(dst);
+    const uint32_t h = umin(((16u - (uint32_t)(reinterpret_cast<uintptr_t>(dst) & 15u)) & 15u) >> 1, nf);
+    if (threadIdx.x < h) d16[threadIdx.x] = (uint16_t)bf16_rne_bits(s[threadIdx.x]);
+    const uint32_t n8 = (nf - h) >> 3;
+    uint4* d = reinterpret_cast<uint4*>(dst + 2 * h);
+    const uint32_t q = h & 3u;
+    const uint4* a = reinterpret_cast<const uint4*>(src + 4 * (h - q));
+    constexpr int kS = 1;  // one block per thread per round: the general get kernel has no registers to spare
+    switch (q) {
+        case 0: cast_blocks_shifted<0, kS>(d, a, n8); break;
+        case 1: cast_blocks_shifted<1, kS>(d, a, n8); break;
+        case 2: cast_blocks_shifted<2, kS>(d, a, n8); break;
+        default: cast_blocks_shifted<3, kS>(d, a, n8); break;
+    }
+    const uint32_t done = h + (n8 << 3);
+    if (threadIdx.x < nf - done) d16[done + threadIdx.x] = (uint16_t)bf16_rne_bits(s[done + threadIdx.x]);
 }
 
 // Largest segment index whose first granule is <= g (segments are non-empty
@@ -502,7 +554,7 @@ __device__ __forceinline__ void run_range(const LaunchParams<BLOB>& p, uint64_t 
                 if (!GENERAL || (reinterpret_cast<uintptr_t>(uaddr) & 15u) == 0)
                     cta_cast_aligned<kV>(uaddr + (off >> 1), paddr, len);
                 else
-                    cta_cast_scalar(uaddr + (off >> 1), paddr, len);
+                    cta_cast_any(uaddr + (off >> 1), paddr, len);
             } else if (!GENERAL || (reinterpret_cast<uintptr_t>(uaddr) & 15u) == 0) {
                 cta_copy_aligned<kV>(uaddr + off, paddr, len);
             } else {

@@ -127,6 +127,39 @@ def test_unaligned_cast_and_copy_kernels():
         assert st.free([int(i)]) == 0
 
 
+def test_cast_into_two_byte_aligned_destinations():
+    """The cast into destinations 2..14 bytes past a 16-byte boundary, for
+    objects of 1 to 70 floats (shorter than, equal to and longer than the
+    aligning head of up to 7 elements, with and without a tail) and one of
+    several 32 KiB pieces, holding every class of value: each output equals
+    the oracle's RNE, and the bytes around it stay untouched."""
+    P = 4096
+    st = store(4096 * P, P)
+    rng = np.random.default_rng(17)
+    special = np.array([0x7F800000, 0xFF800000, 0x7FC00001, 0xFF812345, 0x00000001, 0x80000001, 0x007FFFFF,
+                        0x3F808000, 0x3F818000, 0x7F7FFFFF, 0x00000000, 0x80000000], np.uint32)
+    counts = list(range(1, 18)) + [23, 24, 25, 31, 32, 33, 70, 3 * 8192 + 5]
+    fs = []
+    for k, nf in enumerate(counts):
+        bits = rng.integers(0, 1 << 32, nf, dtype=np.uint64).astype(np.uint32)
+        bits[: min(nf, len(special))] = np.roll(special, k)[: min(nf, len(special))]
+        fs.append(bits)
+    srcs = [torch.from_numpy(b.view(np.uint8).copy()).to(DEV) for b in fs]
+    s, ids = st.put_batch(put_descs(srcs))
+    assert s == 0, st.last_error()
+    for e in range(2, 16, 2):
+        outs = [torch.full((b.size * 2 + 64,), 0xA5, dtype=torch.uint8, device=DEV) for b in fs]
+        s, per = st.get_batch(get_descs([int(i) for i in ids], [o.data_ptr() + 16 + e for o in outs],
+                                        dst_bytes=[b.size * 2 for b in fs], cast=1))
+        assert s == 0 and list(per) == [0] * len(fs), st.last_error()
+        torch.cuda.synchronize()
+        for b, o in zip(fs, outs):
+            h = o.cpu().numpy()
+            lo, hi = 16 + e, 16 + e + 2 * b.size
+            assert np.array_equal(h[lo:hi].view(np.uint16), f32_bits_to_bf16_bits(b)), (e, b.size)
+            assert (h[:lo] == 0xA5).all() and (h[hi:] == 0xA5).all(), (e, b.size)
+
+
 def test_object_larger_than_64_gib():
     """An object of 65 GiB + a ragged tail in 1 GiB pages: its launch byte
     space is split into segments of at most 64 GiB, so 32-bit granule
