@@ -584,11 +584,13 @@ __global__ void __launch_bounds__(kThreads, GENERAL ? kMinBlocksGeneral : kMinBl
     run_share<Mode::Get, GENERAL, BLOB>(p);
 }
 // A get launch without casts: the copy path alone fits the register budget
-// of kMinBlocks resident CTAs, like the put.
-template <int BLOB>
-__global__ void __launch_bounds__(kThreads, kMinBlocks) gather_copy_kernel(const __grid_constant__ LaunchParams<BLOB> p) {
+// of kMinBlocks resident CTAs, like the put (any alignment: the budget of
+// the other general kernels, without the cast's registers).
+template <int BLOB, bool GENERAL>
+__global__ void __launch_bounds__(kThreads, GENERAL ? kMinBlocksGeneral : kMinBlocks)
+    gather_copy_kernel(const __grid_constant__ LaunchParams<BLOB> p) {
     pdl_wait_then_release();
-    run_share<Mode::GetCopy, false, BLOB>(p);
+    run_share<Mode::GetCopy, GENERAL, BLOB>(p);
 }
 template <int BLOB>
 __global__ void __launch_bounds__(kThreads, kMinBlocks) compact_move_kernel(const __grid_constant__ LaunchParams<BLOB> p) {

@@ -14,13 +14,14 @@ t2i_status Store::launch_one(const std::vector<SegDesc>& sd, const std::vector<u
     auto* p = reinterpret_cast<LaunchParams<BLOB>*>(param_buf_);
     const bool chunked =
         uint64_t(n_granules) * kGranule >= kDynMinCtaBytes * uint64_t(max_ctas_[int(M)][GENERAL ? 1 : 0]);
-    // an unchunked get with no cast segment runs the leaner copy-only kernel
-    // (4 resident CTAs per SM instead of 3: +3.8% on the adapter gets; a
-    // chunked get keeps the other kernel, 0.5% faster there)
+    // a get with no cast segment runs the leaner copy-only kernel: aligned
+    // and unchunked (4 resident CTAs per SM instead of 3, +3.8% on the
+    // adapter gets; an aligned chunked get keeps the other kernel, 0.5%
+    // faster there), or any alignment (the cast's registers left out)
     bool any_cast = false;
     for (const SegDesc& d : sd) any_cast = any_cast || (d.nbytes_flags & kCastFlag) != 0;
     const int mode =
-        (M == Mode::Get && !GENERAL && !any_cast && !chunked && kGetCopyKernel) ? int(Mode::GetCopy) : int(M);
+        (M == Mode::Get && !any_cast && (!chunked || GENERAL) && kGetCopyKernel) ? int(Mode::GetCopy) : int(M);
     p->h.pool = pool_;
     p->h.work = chunked ? cur_work_ : 0;
     p->h.chunk_granules = kChunkGranules;
@@ -46,7 +47,7 @@ t2i_status Store::launch_one(const std::vector<SegDesc>& sd, const std::vector<u
     const unsigned grid = static_cast<unsigned>(g);
     void* args[] = {p};
     const void* fn = M == Mode::Put                  ? reinterpret_cast<const void*>(scatter_put_kernel<BLOB, GENERAL>)
-                     : mode == int(Mode::GetCopy)     ? reinterpret_cast<const void*>(gather_copy_kernel<BLOB>)
+                     : mode == int(Mode::GetCopy)     ? reinterpret_cast<const void*>(gather_copy_kernel<BLOB, GENERAL>)
                      : M == Mode::Get                 ? reinterpret_cast<const void*>(gather_get_kernel<BLOB, GENERAL>)
                                                       : reinterpret_cast<const void*>(compact_move_kernel<BLOB>);
     if (fail_countdown_ && --fail_countdown_ == 0) {

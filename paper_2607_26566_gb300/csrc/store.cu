@@ -138,8 +138,8 @@ class Store {
              reinterpret_cast<const void*>(gather_get_kernel<kBlobLarge, true>)},
             {reinterpret_cast<const void*>(compact_move_kernel<kBlobLarge>),
              reinterpret_cast<const void*>(compact_move_kernel<kBlobLarge>)},
-            {reinterpret_cast<const void*>(gather_copy_kernel<kBlobLarge>),
-             reinterpret_cast<const void*>(gather_copy_kernel<kBlobLarge>)}};
+            {reinterpret_cast<const void*>(gather_copy_kernel<kBlobLarge, false>),
+             reinterpret_cast<const void*>(gather_copy_kernel<kBlobLarge, true>)}};
         for (int m = 0; m < 4; ++m)
             for (int a = 0; a < 2; ++a) {
                 int occ = 0;
