@@ -59,6 +59,13 @@ constexpr int kVecPerThread = T2I_TUNE_VEC;         // 16-byte vectors per threa
 constexpr int kMinBlocks = T2I_TUNE_MIN_BLOCKS;     // resident CTAs per SM the register budget must allow
 constexpr int kMinBlocksGet = T2I_TUNE_MIN_BLOCKS_GET;  // same, gather (its cast path needs a few more registers)
 constexpr int kMinBlocksGeneral = 2;  // same, kernels that handle any alignment
+#ifndef T2I_TUNE_MIN_BLOCKS_GENERAL_COPY
+#define T2I_TUNE_MIN_BLOCKS_GENERAL_COPY 3
+#endif
+// same, the any-alignment get without casts (a sweep: 3 resident CTAs per
+// SM, at 80 registers and a few bytes of spill, beat 2 by 17% on unaligned
+// 1 GiB gets; the any-alignment put lost up to 10% at 3, so it keeps 2)
+constexpr int kMinBlocksGeneralCopy = T2I_TUNE_MIN_BLOCKS_GENERAL_COPY;
 constexpr uint32_t kPieceBytes = kThreads * kVecPerThread * 16;  // U = 32 KiB: one round of the copy loop
 constexpr uint32_t kGranule = 32;  // segment starts and CTA shares fall on 32-byte boundaries
 constexpr uint64_t kMinCtaBytes = 16 * 1024;  // smallest share worth a CTA
@@ -584,10 +591,11 @@ __global__ void __launch_bounds__(kThreads, GENERAL ? kMinBlocksGeneral : kMinBl
     run_share<Mode::Get, GENERAL, BLOB>(p);
 }
 // A get launch without casts: the copy path alone fits the register budget
-// of kMinBlocks resident CTAs, like the put (any alignment: the budget of
-// the other general kernels, without the cast's registers).
+// of kMinBlocks resident CTAs, like the put (any alignment: 3 resident CTAs
+// per SM, one more than the other general kernels, without the cast's
+// registers).
 template <int BLOB, bool GENERAL>
-__global__ void __launch_bounds__(kThreads, GENERAL ? kMinBlocksGeneral : kMinBlocks)
+__global__ void __launch_bounds__(kThreads, GENERAL ? kMinBlocksGeneralCopy : kMinBlocks)
     gather_copy_kernel(const __grid_constant__ LaunchParams<BLOB> p) {
     pdl_wait_then_release();
     run_share<Mode::GetCopy, GENERAL, BLOB>(p);
