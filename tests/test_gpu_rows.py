@@ -12,7 +12,8 @@ import torch
 
 import bench
 import workloads as W
-from oracle import EVICTED, OK, OracleStore, PutItem
+from adapter_replay import AdapterShapes, OracleBackend, Replay
+from oracle import OK, OracleStore, PutItem
 
 pytestmark = pytest.mark.gpu
 DEV = torch.device("cuda", 0)
@@ -89,43 +90,15 @@ def test_compaction_full_size():
     cp.close()
 
 
-class OracleAdapters:
-    """The adapter harness's decisions replayed on the oracle (metadata only):
-    the same reload-only-the-missing rule, driven by the oracle's victims."""
-
-    def __init__(self, ad: "bench.Adapters"):
-        self.ad = ad
-        self.ora = OracleStore(ad.pool.numel(), W.ADAPTERS["page_bytes"], keep_bytes=False)
-        self.ids, self.missing, self.owner = {}, {}, {}
-        self.victims = []
-
-    def load(self, s):
-        r = int(self.ad.ranks[s])
-        if s not in self.ids:
-            js = list(range(len(self.ad.sizes[r])))
-            self.ids[s] = [0] * len(js)
-        else:
-            js = sorted(self.missing.get(s, ()))
-            if not js:
-                return
-        st, ids = self.ora.put_batch([PutItem(int(self.ad.sizes[r][j]), None, W.DTYPE_BF16, s,
-                                              int(self.ad.blocks[r][j]), True) for j in js])
-        assert st == OK
-        for j, i in zip(js, ids):
-            self.ids[s][j] = i
-            self.owner[i] = (s, j)
-        self.missing[s] = set()
-        for v in self.ora.last_evictions:
-            s2, j2 = self.owner.pop(v)
-            self.missing.setdefault(s2, set()).add(j2)
-            self.victims.append(v)
-
-    def call(self, k):
-        s, w = int(self.ad.sets[k]), int(self.ad.starts[k])
-        if s not in self.ids or any(w <= j < w + self.ad.window for j in self.missing.get(s, ())):
-            self.load(s)
-        st, _, _ = self.ora.get_batch(self.ids[s][w:w + self.ad.window])
-        assert st == OK
+def _oracle_replay(ad: "bench.Adapters", n_calls: int) -> Replay:
+    """The harness's decisions on the same draws, replayed on the oracle's
+    paged model (metadata only)."""
+    sh = AdapterShapes(n_sets=len(ad.ranks), n_calls=len(ad.sets), window=ad.window)
+    assert np.array_equal(sh.sets, ad.sets) and np.array_equal(sh.starts, ad.starts)
+    rep = Replay(sh, OracleBackend(ad.pool.numel(), W.ADAPTERS["page_bytes"]))
+    for k in range(n_calls):
+        rep.call(k)
+    return rep
 
 
 def test_adapters_small_vs_oracle():
@@ -133,7 +106,8 @@ def test_adapters_small_vs_oracle():
     victims in the same order, the same page lists; every got window equals
     its bank bytes."""
     ad = bench.Adapters(DEV, n_sets=64, n_calls=400, pool_bytes=2 << 30)
-    oa = OracleAdapters(ad)
+    sh = AdapterShapes(n_sets=64, n_calls=400)
+    oa = Replay(sh, OracleBackend(ad.pool.numel(), W.ADAPTERS["page_bytes"]))
     for k in range(400):
         s, w = ad.call(k)
         oa.call(k)
@@ -141,24 +115,35 @@ def test_adapters_small_vs_oracle():
         n = ad.expected(s, w).numel()
         assert torch.equal(ad.dst[:n], ad.expected(s, w)), k
     assert ad.victims and ad.loads > 64          # evictions and partial reloads happened
+    assert ad.loads == oa.loads
     for s, ids in oa.ids.items():
         for oid in ids[::50]:
-            o = oa.ora.objects.get(int(oid))
+            o = oa.b.ora.objects.get(int(oid))
             if o is not None:
                 assert ad.store.ctl.object(int(oid))[2] == o.pages
-    assert ad.store.ctl.free_pages() == oa.ora.free_stack
+    assert ad.store.ctl.free_pages() == oa.b.free_pages()
     ad.close()
 
 
-def test_adapters_full_size_windows():
-    """The full adapter workload (512 sets, 16 GiB pool), 3,000 calls; every
-    50th window compared with its bank bytes."""
-    ad = bench.Adapters(DEV, n_calls=3000)
-    for k in range(3000):
+def test_adapters_full_size_vs_oracle():
+    """The full adapter workload (512 sets, 16 GiB pool, 256 KiB pages), its
+    first 3,000 calls on the GPU store: the store evicts exactly the oracle's
+    victims in the oracle's order, reloads as often, and ends with the
+    oracle's free-page stack; every 50th window equals its bank bytes. (All
+    10,000 calls of the trace are replayed on the control core against the
+    oracle in the CPU tests.)"""
+    n = 3000
+    ad = bench.Adapters(DEV, n_calls=n)
+    for k in range(n):
         s, w = ad.call(k)
         if k % 50 == 0:
-            n = ad.expected(s, w).numel()
-            assert torch.equal(ad.dst[:n], ad.expected(s, w)), k
+            m = ad.expected(s, w).numel()
+            assert torch.equal(ad.dst[:m], ad.expected(s, w)), k
+    oa = _oracle_replay(ad, n)
+    assert len(ad.victims) == len(oa.victims) > 100_000
+    assert ad.victims == oa.victims
+    assert ad.loads == oa.loads
+    assert ad.store.ctl.free_pages() == oa.b.free_pages()
     st = ad.store.stats()
-    assert st["evictions"] > 0 and st["used_pages"] <= st["limit_pages"]
+    assert st["evictions"] == len(oa.victims) and st["used_pages"] <= st["limit_pages"]
     ad.close()

@@ -218,8 +218,8 @@ def test_handoff_small_vs_oracle():
 def test_handoff_full_size(B):
     """8 GiB pool, 2 MiB pages, 64 requests in flight, the launch shape the
     benchmark times. Every non-cast get must equal its input byte for byte
-    (get(put(x)) == x); the cast latents of 8 sampled requests (all at B = 1)
-    are compared with the oracle's RNE."""
+    (get(put(x)) == x), and every request's cast latents must equal the
+    oracle's RNE of its input."""
     C = W.HANDOFF
     specs = W.handoff_specs(B)
     st = make_store(C["pool_bytes"], C["page_bytes"])
@@ -235,7 +235,6 @@ def test_handoff_full_size(B):
         reqs.append(ts)
         ids_all.append(oids)
     compare_meta(st, ora)
-    sampled = set(range(C["requests"])) if B == 1 else set(range(0, C["requests"], 8))
     for r, (ts, oids) in enumerate(zip(reqs, ids_all)):
         outs = [torch.empty_like(t) if j != ci else torch.empty(t.shape, dtype=torch.bfloat16, device=DEV)
                 for j, t in enumerate(ts)]
@@ -246,10 +245,9 @@ def test_handoff_full_size(B):
         for j, (t, o) in enumerate(zip(ts, outs)):
             if j != ci:
                 assert torch.equal(t.view(torch.uint8).reshape(-1), o.view(torch.uint8).reshape(-1)), (r, j)
-        if r in sampled:
-            lat = ts[ci].reshape(-1).view(torch.int32).cpu().numpy().view(np.uint32)
-            got = outs[ci].reshape(-1).view(torch.int16).cpu().numpy().view(np.uint16)
-            assert np.array_equal(got, f32_bits_to_bf16_bits(lat)), r
+        lat = ts[ci].reshape(-1).view(torch.int32).cpu().numpy().view(np.uint32)
+        got = outs[ci].reshape(-1).view(torch.int16).cpu().numpy().view(np.uint16)
+        assert np.array_equal(got, f32_bits_to_bf16_bits(lat)), r
     for oids in ids_all:
         assert st.free(oids) == 0
     assert st.stats()["used_pages"] == 0
