@@ -338,9 +338,11 @@ t2i_status t2i_inject_launch_failure(t2i_store* store, uint32_t countdown);
  * ========================================================================= */
 
 /* Copies one object's pages out of a pool into a contiguous device buffer,
- * as a one-item t2i_get_batch does (the same gather kernel, the same bytes,
- * the same optional fp32 -> bf16 RNE cast), but with no store and without
- * allocating any memory.
+ * with the same bytes and the same optional fp32 -> bf16 RNE cast as a
+ * one-item t2i_get_batch, but with no store and without allocating any
+ * memory. Its launches are those of a store's chunked get: the cast-capable
+ * gather kernel for a 16-byte aligned destination or a cast, the copy-only
+ * gather kernel for any other destination.
  *
  * Who needs it: a caller that must not allocate device memory while it
  * moves data. In a serving process the free HBM is often reserved up front

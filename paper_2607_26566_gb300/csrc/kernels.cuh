@@ -26,7 +26,8 @@
 // HBM-bound by construction (2 bytes of traffic per payload byte, 1.5 for the
 // cast): fully coalesced 16-byte accesses, enough bytes in flight per SM (8
 // independent 16-byte loads per thread before the first store, 3-4 resident
-// CTAs of 256 threads per SM: 96-128 KiB in flight), grids sized from the SM
+// CTAs of 256 threads per SM: 96-128 KiB in flight; user addresses that are
+// not 16-byte aligned are realigned in shared memory), grids sized from the SM
 // count, the occupancy and the launch's bytes (see the work split above), and
 // programmatic dependent launch so that the next launch's set-up overlaps the
 // end of this one. The launch shape and cache policy were chosen by a sweep
@@ -58,14 +59,20 @@ constexpr int kThreads = T2I_TUNE_THREADS;          // threads per CTA
 constexpr int kVecPerThread = T2I_TUNE_VEC;         // 16-byte vectors per thread per round of a copy loop
 constexpr int kMinBlocks = T2I_TUNE_MIN_BLOCKS;     // resident CTAs per SM the register budget must allow
 constexpr int kMinBlocksGet = T2I_TUNE_MIN_BLOCKS_GET;  // same, gather (its cast path needs a few more registers)
-constexpr int kMinBlocksGeneral = 2;  // same, kernels that handle any alignment
-#ifndef T2I_TUNE_MIN_BLOCKS_GENERAL_COPY
-#define T2I_TUNE_MIN_BLOCKS_GENERAL_COPY 3
+#ifndef T2I_TUNE_MIN_BLOCKS_GENERAL
+#define T2I_TUNE_MIN_BLOCKS_GENERAL 3
 #endif
-// same, the any-alignment get without casts (a sweep: 3 resident CTAs per
-// SM, at 80 registers and a few bytes of spill, beat 2 by 17% on unaligned
-// 1 GiB gets; the any-alignment put lost up to 10% at 3, so it keeps 2)
-constexpr int kMinBlocksGeneralCopy = T2I_TUNE_MIN_BLOCKS_GENERAL_COPY;
+// same, the any-alignment kernels (their pieces are staged in shared memory,
+// 32 KiB per CTA, so that their loads need no more registers than the
+// aligned kernels'). A sweep over 1 GiB at misaligned offsets: 3 resident
+// CTAs per SM beat 4 by 1-2% on copies and by 12% on the cast into 2-byte
+// aligned destinations; 5 lost 5-12%.
+constexpr int kMinBlocksGeneral = T2I_TUNE_MIN_BLOCKS_GENERAL;
+#ifndef T2I_TUNE_MIN_BLOCKS_GENERAL_GET
+#define T2I_TUNE_MIN_BLOCKS_GENERAL_GET T2I_TUNE_MIN_BLOCKS_GENERAL
+#endif
+// same, the any-alignment get that may cast
+constexpr int kMinBlocksGeneralGet = T2I_TUNE_MIN_BLOCKS_GENERAL_GET;
 constexpr uint32_t kPieceBytes = kThreads * kVecPerThread * 16;  // U = 32 KiB: one round of the copy loop
 constexpr uint32_t kGranule = 32;  // segment starts and CTA shares fall on 32-byte boundaries
 constexpr uint64_t kMinCtaBytes = 16 * 1024;  // smallest share worth a CTA
@@ -262,62 +269,6 @@ __device__ __noinline__ void cta_copy_pages(unsigned char* __restrict__ user, un
     }
 }
 
-// dst 16-byte aligned, src misaligned by sm (1..15): each output vector is
-// cut out of the two aligned source vectors that cover it. Both aligned
-// loads hold at least one byte of the source range, so no access leaves the
-// source allocation.
-template <int Q>
-__device__ __forceinline__ void cta_copy_shifted_q(uint4* __restrict__ d, const uint4* __restrict__ a,
-                                                   uint32_t nvec, uint32_t r) {
-    // two aligned loads per output vector; a fixed 2 vectors per round keeps
-    // this rare path within the register budget of the general kernels
-    constexpr int kV = 2;
-#pragma unroll 1
-    for (uint32_t base = 0; base < nvec; base += kThreads * kV) {
-        uint4 lo[kV], hi[kV];
-#pragma unroll
-        for (int j = 0; j < kV; ++j) {
-            const uint32_t v = base + j * kThreads + threadIdx.x;
-            if (v < nvec) {
-                lo[j] = ld_stream(a + v);
-                hi[j] = ld_stream(a + v + 1);
-            }
-        }
-#pragma unroll
-        for (int j = 0; j < kV; ++j) {
-            const uint32_t v = base + j * kThreads + threadIdx.x;
-            if (v < nvec) st_stream(d + v, shift_pick<Q>(lo[j], hi[j], r));
-        }
-    }
-}
-
-__device__ __forceinline__ void cta_copy_unaligned(unsigned char* __restrict__ dst, const unsigned char* __restrict__ src,
-                                                uint32_t len) {
-    // head bytes up to dst's 16-byte boundary
-    const uint32_t head = umin(len, (16u - (uint32_t)(reinterpret_cast<uintptr_t>(dst) & 15u)) & 15u);
-    if (threadIdx.x < head) dst[threadIdx.x] = src[threadIdx.x];
-    dst += head;
-    src += head;
-    len -= head;
-    const uint32_t nvec = len >> 4;
-    const uint32_t sm = (uint32_t)(reinterpret_cast<uintptr_t>(src) & 15u);
-    if (sm == 0) {
-        cta_copy_aligned<kVecPerThread / 2>(dst, src, len);
-        return;
-    }
-    uint4* d = reinterpret_cast<uint4*>(dst);
-    const uint4* a = reinterpret_cast<const uint4*>(src - sm);
-    const uint32_t r = sm & 3u;
-    switch (sm >> 2) {
-        case 0: cta_copy_shifted_q<0>(d, a, nvec, r); break;
-        case 1: cta_copy_shifted_q<1>(d, a, nvec, r); break;
-        case 2: cta_copy_shifted_q<2>(d, a, nvec, r); break;
-        default: cta_copy_shifted_q<3>(d, a, nvec, r); break;
-    }
-    const uint32_t tail = len & 15u;
-    if (threadIdx.x < tail) dst[(nvec << 4) + threadIdx.x] = src[(nvec << 4) + threadIdx.x];
-}
-
 // fp32 (pool, aligned) -> bf16 (user, 16-byte aligned). len = source
 // bytes, a multiple of 4: 8 floats (two 16-byte loads) -> 8 bf16 (one
 // 16-byte store) per thread step, the last < 8 elements one by one.
@@ -360,67 +311,132 @@ __device__ __forceinline__ void cta_cast_aligned(unsigned char* __restrict__ dst
     }
 }
 
-// Blocks of 8 floats whose words start Q (0..3) words past the aligned
-// vectors a[2v]: each is cut out of a[2v], a[2v+1] and (Q > 0) a[2v+2],
-// cast, and stored as one 16-byte vector d[v]. Every aligned load holds at
-// least one word of the block, so no access leaves the source allocation.
-template <int Q, int S>
-__device__ __forceinline__ void cast_blocks_shifted(uint4* __restrict__ d, const uint4* __restrict__ a, uint32_t n8) {
-#pragma unroll 1
-    for (uint32_t base = 0; base < n8; base += kThreads * S) {
-        uint4 x[S], y[S], z[S];
+// ------------------------------------------------ any alignment: staged copies
+// The any-alignment kernels stage each piece in shared memory: the aligned
+// 16-byte window that covers the piece's source bytes is loaded with
+// independent aligned 16-byte loads (kVecPerThread per thread, all issued
+// before the first is used), then every aligned 16-byte output vector is
+// cut out of the staged window (two staged vectors and funnel shifts), so
+// every global access is one aligned 16-byte vector and the loads in flight
+// per SM are those of the aligned kernels. Each aligned load holds at least
+// one byte of the source range, so no access leaves the source allocation.
+// A piece is at most U bytes, so its window (up to 15 bytes of misalignment
+// in front) is at most U/16 + 1 vectors: one round of kVecPerThread loads
+// per thread, plus one more vector.
+constexpr uint32_t kStageVecs = kPieceBytes / 16 + 1;
+static_assert(kThreads * kVecPerThread * 16 == kPieceBytes, "one round of loads per piece");
+// The stage of a CTA of the any-alignment kernels (only they reference it).
+__shared__ uint4 g_stage[kStageVecs];
+
+// Loads the nw <= kStageVecs aligned vectors at a into stage, then a CTA
+// barrier (every thread sees the whole window).
+__device__ __forceinline__ void stage_window(uint4* __restrict__ stage, const uint4* __restrict__ a, uint32_t nw) {
+    constexpr uint32_t kRound = kThreads * kVecPerThread;
+    uint4 r[kVecPerThread];
 #pragma unroll
-        for (int j = 0; j < S; ++j) {
-            const uint32_t v = base + j * kThreads + threadIdx.x;
-            if (v < n8) {
-                x[j] = ld_stream(a + 2 * v);
-                y[j] = ld_stream(a + 2 * v + 1);
-                if (Q > 0) z[j] = ld_stream(a + 2 * v + 2);
-            }
-        }
+    for (int j = 0; j < kVecPerThread; ++j) {
+        const uint32_t v = j * kThreads + threadIdx.x;
+        if (v < nw) r[j] = ld_stream(a + v);
+    }
+    const bool extra = kRound + threadIdx.x < nw;  // the window's last vector, past one round
+    uint4 x;
+    if (extra) x = ld_stream(a + kRound + threadIdx.x);
 #pragma unroll
-        for (int j = 0; j < S; ++j) {
-            const uint32_t v = base + j * kThreads + threadIdx.x;
-            if (v < n8) {
-                const uint32_t w[12] = {x[j].x, x[j].y, x[j].z, x[j].w, y[j].x, y[j].y,
-                                        y[j].z, y[j].w, Q > 0 ? z[j].x : 0u, Q > 0 ? z[j].y : 0u,
-                                        Q > 0 ? z[j].z : 0u, 0u};
-                uint4 o;
-                o.x = pack_bf16x2(w[Q + 0], w[Q + 1]);
-                o.y = pack_bf16x2(w[Q + 2], w[Q + 3]);
-                o.z = pack_bf16x2(w[Q + 4], w[Q + 5]);
-                o.w = pack_bf16x2(w[Q + 6], w[Q + 7]);
-                st_stream(d + v, o);
-            }
-        }
+    for (int j = 0; j < kVecPerThread; ++j) {
+        const uint32_t v = j * kThreads + threadIdx.x;
+        if (v < nw) stage[v] = r[j];
+    }
+    if (extra) stage[kRound + threadIdx.x] = x;
+    __syncthreads();
+}
+
+// Output vectors d[v] = bytes [16 v + 4 Q + r, ... + 16) of the staged
+// window w (r in 0..3; Q = r = 0 is a plain copy).
+template <int Q>
+__device__ __forceinline__ void emit_shifted(uint4* __restrict__ d, const uint4* __restrict__ w, uint32_t nvec,
+                                             uint32_t r) {
+#pragma unroll 4
+    for (uint32_t v = threadIdx.x; v < nvec; v += kThreads) {
+        if (Q == 0 && r == 0)
+            st_stream(d + v, w[v]);
+        else
+            st_stream(d + v, shift_pick<Q>(w[v], w[v + 1], r));
     }
 }
 
-// Same cast into a destination that is only 2-byte aligned. The first
-// h < 8 elements, one per thread, bring the destination to a 16-byte
-// boundary; the source (16-byte aligned) is then h words past one, so the
-// blocks of 8 are cut out of aligned loads (cast_blocks_shifted); the last
-// < 8 elements one per thread.
-__device__ __forceinline__ void cta_cast_any(unsigned char* __restrict__ dst, const unsigned char* __restrict__ src,
+// CTA-wide copy of len <= U bytes, any alignment on either
+// side: stage the source window, then the destination's head bytes (up to
+// its 16-byte boundary) one per thread, its aligned vectors, and the tail
+// bytes one per thread.
+__device__ __noinline__ void cta_copy_staged(unsigned char* __restrict__ dst, const unsigned char* __restrict__ src,
                                              uint32_t len) {
+    uint4* stage = g_stage;
+    const uint32_t s0 = (uint32_t)(reinterpret_cast<uintptr_t>(src) & 15u);
+    stage_window(stage, reinterpret_cast<const uint4*>(src - s0), (s0 + len + 15) >> 4);
+    const unsigned char* wb = reinterpret_cast<const unsigned char*>(stage);
+    const uint32_t head = umin(len, (16u - (uint32_t)(reinterpret_cast<uintptr_t>(dst) & 15u)) & 15u);
+    if (threadIdx.x < head) dst[threadIdx.x] = wb[s0 + threadIdx.x];
+    const uint32_t s = s0 + head;  // window offset of the first aligned output vector (< 32)
+    const uint32_t nvec = (len - head) >> 4;
+    uint4* d = reinterpret_cast<uint4*>(dst + head);
+    const uint4* w = stage + (s >> 4);
+    const uint32_t r = s & 3u;
+    switch ((s >> 2) & 3u) {
+        case 0: emit_shifted<0>(d, w, nvec, r); break;
+        case 1: emit_shifted<1>(d, w, nvec, r); break;
+        case 2: emit_shifted<2>(d, w, nvec, r); break;
+        default: emit_shifted<3>(d, w, nvec, r); break;
+    }
+    const uint32_t done = head + (nvec << 4);
+    if (threadIdx.x < len - done) dst[done + threadIdx.x] = wb[s0 + done + threadIdx.x];
+    __syncthreads();  // the stage is free for the next piece
+}
+
+// Blocks of 8 staged floats starting Q (0..3) words past the staged vectors
+// a[2v]: each is cut out of a[2v], a[2v+1] and (Q > 0) a[2v+2], cast, and
+// stored as one 16-byte vector d[v].
+template <int Q>
+__device__ __forceinline__ void emit_cast_blocks(uint4* __restrict__ d, const uint4* __restrict__ a, uint32_t n8) {
+#pragma unroll 1
+    for (uint32_t v = threadIdx.x; v < n8; v += kThreads) {
+        const uint4 x = a[2 * v], y = a[2 * v + 1];
+        const uint4 z = Q > 0 ? a[2 * v + 2] : make_uint4(0u, 0u, 0u, 0u);
+        const uint32_t w[12] = {x.x, x.y, x.z, x.w, y.x, y.y, y.z, y.w, z.x, z.y, z.z, z.w};
+        uint4 o;
+        o.x = pack_bf16x2(w[Q + 0], w[Q + 1]);
+        o.y = pack_bf16x2(w[Q + 2], w[Q + 3]);
+        o.z = pack_bf16x2(w[Q + 4], w[Q + 5]);
+        o.w = pack_bf16x2(w[Q + 6], w[Q + 7]);
+        st_stream(d + v, o);
+    }
+}
+
+// fp32 (pool, 16-byte aligned) -> bf16 into a destination that is 2-byte
+// aligned, len <= U source bytes (a multiple of 4): stage
+// the source, then the first h < 8 elements one per thread (they bring the
+// destination to a 16-byte boundary), blocks of 8 as 16-byte stores, and
+// the last < 8 elements one per thread.
+__device__ __noinline__ void cta_cast_staged(unsigned char* __restrict__ dst, const unsigned char* __restrict__ src,
+                                             uint32_t len) {
+    uint4* stage = g_stage;
+    stage_window(stage, reinterpret_cast<const uint4*>(src), (len + 15) >> 4);
+    const uint32_t* ws = reinterpret_cast<const uint32_t*>(stage);
     const uint32_t nf = len >> 2;
-    const uint32_t* s = reinterpret_cast<const uint32_t*>(src);
     uint16_t* d16 = reinterpret_cast<uint16_t*>(dst);
     const uint32_t h = umin(((16u - (uint32_t)(reinterpret_cast<uintptr_t>(dst) & 15u)) & 15u) >> 1, nf);
-    if (threadIdx.x < h) d16[threadIdx.x] = (uint16_t)bf16_rne_bits(s[threadIdx.x]);
+    if (threadIdx.x < h) d16[threadIdx.x] = (uint16_t)bf16_rne_bits(ws[threadIdx.x]);
     const uint32_t n8 = (nf - h) >> 3;
     uint4* d = reinterpret_cast<uint4*>(dst + 2 * h);
-    const uint32_t q = h & 3u;
-    const uint4* a = reinterpret_cast<const uint4*>(src + 4 * (h - q));
-    constexpr int kS = 1;  // one block per thread per round: the general get kernel has no registers to spare
-    switch (q) {
-        case 0: cast_blocks_shifted<0, kS>(d, a, n8); break;
-        case 1: cast_blocks_shifted<1, kS>(d, a, n8); break;
-        case 2: cast_blocks_shifted<2, kS>(d, a, n8); break;
-        default: cast_blocks_shifted<3, kS>(d, a, n8); break;
+    const uint4* a = stage + (h >> 2);
+    switch (h & 3u) {
+        case 0: emit_cast_blocks<0>(d, a, n8); break;
+        case 1: emit_cast_blocks<1>(d, a, n8); break;
+        case 2: emit_cast_blocks<2>(d, a, n8); break;
+        default: emit_cast_blocks<3>(d, a, n8); break;
     }
     const uint32_t done = h + (n8 << 3);
-    if (threadIdx.x < nf - done) d16[done + threadIdx.x] = (uint16_t)bf16_rne_bits(s[done + threadIdx.x]);
+    if (threadIdx.x < nf - done) d16[done + threadIdx.x] = (uint16_t)bf16_rne_bits(ws[done + threadIdx.x]);
+    __syncthreads();  // the stage is free for the next piece
 }
 
 // Largest segment index whose first granule is <= g (segments are non-empty
@@ -447,9 +463,8 @@ __device__ __forceinline__ void pdl_wait_then_release() {
 
 // The piece loop. GENERAL = false: every user address of the launch is
 // 16-byte aligned (the host sorts segments into aligned and other launches),
-// so only the vector paths are compiled in and the register budget stays
-// small enough for kMinBlocks resident CTAs per SM. GENERAL = true adds the
-// shifted copies and the element-wise cast for any alignment.
+// so the pieces are plain vector copies. GENERAL = true: user addresses of
+// any alignment; every piece is staged in shared memory and realigned there.
 template <Mode M, bool GENERAL, int BLOB>
 __device__ __forceinline__ void run_range(const LaunchParams<BLOB>& p, uint64_t g0, uint64_t g1);
 
@@ -498,9 +513,7 @@ __device__ __forceinline__ void run_share(const LaunchParams<BLOB>& p) {
 // Copies granules [g0, g1) of the launch byte space.
 template <Mode M, bool GENERAL, int BLOB>
 __device__ __forceinline__ void run_range(const LaunchParams<BLOB>& p, uint64_t g0, uint64_t g1) {
-    // the general kernels run at 2 CTAs/SM with room for the shifted paths:
-    // they take half the vectors per round (a piece is then two rounds)
-    constexpr int kV = GENERAL ? kVecPerThread / 2 : kVecPerThread;
+    constexpr int kV = kVecPerThread;
     const SegDesc* segs = reinterpret_cast<const SegDesc*>(p.blob);
     const uint32_t* pages = reinterpret_cast<const uint32_t*>(p.blob + p.h.pages_offset);
     unsigned char* pool = reinterpret_cast<unsigned char*>(p.h.pool);
@@ -533,9 +546,8 @@ __device__ __forceinline__ void run_range(const LaunchParams<BLOB>& p, uint64_t 
         // this segment, each vector finding its own page, instead of
         // stopping at every page end (+2% on a handoff in 16 and 64 KiB pages)
         constexpr uint64_t kRound = uint64_t(kThreads) * kV * 16;
-        if (pmask + 1 < kRound && off + kRound <= nbytes && pos + kRound <= end &&
-            !(s.nbytes_flags & (kCastFlag | kRunFlag)) &&
-            (!GENERAL || (reinterpret_cast<uintptr_t>(s.user) & 15u) == 0)) {
+        if (!GENERAL && pmask + 1 < kRound && off + kRound <= nbytes && pos + kRound <= end &&
+            !(s.nbytes_flags & (kCastFlag | kRunFlag))) {
             cta_copy_pages<M, kV>(reinterpret_cast<unsigned char*>(s.user), pool, pages + s.page_begin, off, pshift);
             pos += kRound;
             continue;
@@ -558,20 +570,20 @@ __device__ __forceinline__ void run_range(const LaunchParams<BLOB>& p, uint64_t 
         unsigned char* uaddr = reinterpret_cast<unsigned char*>(s.user);
         if (M == Mode::Get || M == Mode::GetCopy) {
             if (M == Mode::Get && (s.nbytes_flags & kCastFlag)) {
-                if (!GENERAL || (reinterpret_cast<uintptr_t>(uaddr) & 15u) == 0)
-                    cta_cast_aligned<kV>(uaddr + (off >> 1), paddr, len);
+                if (GENERAL)
+                    cta_cast_staged(uaddr + (off >> 1), paddr, len);
                 else
-                    cta_cast_any(uaddr + (off >> 1), paddr, len);
-            } else if (!GENERAL || (reinterpret_cast<uintptr_t>(uaddr) & 15u) == 0) {
-                cta_copy_aligned<kV>(uaddr + off, paddr, len);
+                    cta_cast_aligned<kV>(uaddr + (off >> 1), paddr, len);
+            } else if (GENERAL) {
+                cta_copy_staged(uaddr + off, paddr, len);
             } else {
-                cta_copy_unaligned(uaddr + off, paddr, len);
+                cta_copy_aligned<kV>(uaddr + off, paddr, len);
             }
         } else {
-            if (!GENERAL || (reinterpret_cast<uintptr_t>(uaddr) & 15u) == 0)
-                cta_copy_aligned<kV>(paddr, uaddr + off, len);
+            if (GENERAL)
+                cta_copy_staged(paddr, uaddr + off, len);
             else
-                cta_copy_unaligned(paddr, uaddr + off, len);
+                cta_copy_aligned<kV>(paddr, uaddr + off, len);
         }
         pos += len;
     }
@@ -585,17 +597,15 @@ __global__ void __launch_bounds__(kThreads, GENERAL ? kMinBlocksGeneral : kMinBl
     run_share<Mode::Put, GENERAL, BLOB>(p);
 }
 template <int BLOB, bool GENERAL>
-__global__ void __launch_bounds__(kThreads, GENERAL ? kMinBlocksGeneral : kMinBlocksGet)
+__global__ void __launch_bounds__(kThreads, GENERAL ? kMinBlocksGeneralGet : kMinBlocksGet)
     gather_get_kernel(const __grid_constant__ LaunchParams<BLOB> p) {
     pdl_wait_then_release();
     run_share<Mode::Get, GENERAL, BLOB>(p);
 }
 // A get launch without casts: the copy path alone fits the register budget
-// of kMinBlocks resident CTAs, like the put (any alignment: 3 resident CTAs
-// per SM, one more than the other general kernels, without the cast's
-// registers).
+// of kMinBlocks resident CTAs, like the put (the cast's registers left out).
 template <int BLOB, bool GENERAL>
-__global__ void __launch_bounds__(kThreads, GENERAL ? kMinBlocksGeneralCopy : kMinBlocks)
+__global__ void __launch_bounds__(kThreads, GENERAL ? kMinBlocksGeneral : kMinBlocks)
     gather_copy_kernel(const __grid_constant__ LaunchParams<BLOB> p) {
     pdl_wait_then_release();
     run_share<Mode::GetCopy, GENERAL, BLOB>(p);

@@ -12,14 +12,17 @@ template <Mode M, bool GENERAL, int BLOB>
 t2i_status Store::launch_one(const std::vector<SegDesc>& sd, const std::vector<uint32_t>& pages, uint32_t n_granules,
                              cudaStream_t stream) {
     auto* p = reinterpret_cast<LaunchParams<BLOB>*>(param_buf_);
-    const bool chunked =
-        uint64_t(n_granules) * kGranule >= kDynMinCtaBytes * uint64_t(max_ctas_[int(M)][GENERAL ? 1 : 0]);
     // a get with no cast segment runs the leaner copy-only kernel: aligned
     // and unchunked (4 resident CTAs per SM instead of 3, +3.8% on the
     // adapter gets; an aligned chunked get keeps the other kernel, 0.5%
     // faster there), or any alignment (the cast's registers left out)
     bool any_cast = false;
     for (const SegDesc& d : sd) any_cast = any_cast || (d.nbytes_flags & kCastFlag) != 0;
+    // chunks from the counter when the launch holds at least kDynMinCtaBytes
+    // per resident CTA of the kernel that would run chunked
+    const bool copy_any = M == Mode::Get && !any_cast && GENERAL && kGetCopyKernel;
+    const bool chunked = uint64_t(n_granules) * kGranule >=
+                         kDynMinCtaBytes * uint64_t(max_ctas_[copy_any ? int(Mode::GetCopy) : int(M)][GENERAL ? 1 : 0]);
     const int mode =
         (M == Mode::Get && !any_cast && (!chunked || GENERAL) && kGetCopyKernel) ? int(Mode::GetCopy) : int(M);
     p->h.pool = pool_;

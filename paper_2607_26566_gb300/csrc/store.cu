@@ -1040,14 +1040,25 @@ static __device__ __align__(256) t2i::WorkCounter t2i_noalloc_scratch[t2i::kNoAl
 namespace t2i {
 namespace {
 
+// The kernels a call can run, as a store's chunked get picks them: the
+// cast-capable gather for 16-byte aligned destinations and for casts, the
+// copy-only gather for other destinations without a cast.
+enum NoAllocKernel { kNoAllocGetAligned = 0, kNoAllocGetAny = 1, kNoAllocCopyAny = 2 };
+
 // Per-device set-up, done once by the first call on that device: the
 // device address of the scratch array (host code sees only a stand-in for
 // the symbol) and the resident CTAs of the gather kernels (its grid size).
 struct NoAllocDevice {
     bool ready = false;
     WorkCounter* scratch = nullptr;
-    int max_ctas[2] = {1, 1};  // [any alignment]
+    int max_ctas[3] = {1, 1, 1};  // [NoAllocKernel]
 };
+
+const void* noalloc_kernel(int k) {
+    return k == kNoAllocGetAligned ? reinterpret_cast<const void*>(gather_get_kernel<kBlobLarge, false>)
+           : k == kNoAllocGetAny   ? reinterpret_cast<const void*>(gather_get_kernel<kBlobLarge, true>)
+                                   : reinterpret_cast<const void*>(gather_copy_kernel<kBlobLarge, true>);
+}
 
 std::mutex g_noalloc_mu;
 NoAllocDevice g_noalloc_dev[kNoAllocMaxDevices];
@@ -1069,11 +1080,9 @@ t2i_status noalloc_setup(int device, NoAllocDevice** out) {
             set_thread_error("t2i_gather_noalloc: cannot query the device");
             return T2I_ERR_CUDA;
         }
-        const void* fns[2] = {reinterpret_cast<const void*>(gather_get_kernel<kBlobLarge, false>),
-                              reinterpret_cast<const void*>(gather_get_kernel<kBlobLarge, true>)};
-        for (int k = 0; k < 2; ++k) {
+        for (int k = 0; k < 3; ++k) {
             int occ = 0;
-            cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, fns[k], kThreads, 0);
+            cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, noalloc_kernel(k), kThreads, 0);
             d.max_ctas[k] = sms * (occ > 0 ? occ : 1);
         }
         d.scratch = static_cast<WorkCounter*>(ptr);
@@ -1083,20 +1092,11 @@ t2i_status noalloc_setup(int device, NoAllocDevice** out) {
     return T2I_OK;
 }
 
-template <bool GENERAL, int BLOB>
-cudaError_t noalloc_launch(const LaunchParams<BLOB>& p, unsigned grid, cudaStream_t stream) {
-    cudaLaunchConfig_t lc = {};
-    lc.gridDim = dim3(grid);
-    lc.blockDim = dim3(kThreads);
-    lc.stream = stream;
-    void* args[] = {const_cast<LaunchParams<BLOB>*>(&p)};
-    return cudaLaunchKernelExC(&lc, reinterpret_cast<const void*>(gather_get_kernel<BLOB, GENERAL>), args);
-}
-
-// One launch: `np` pages of the object starting at page index `p0`.
-template <bool GENERAL>
-t2i_status noalloc_one(const NoAllocDevice& d, uint32_t k, const void* pool, int shift, const uint32_t* pages,
-                       uint64_t p0, uint64_t np, uint64_t nbytes, unsigned char* dst, bool cast, cudaStream_t stream) {
+// One launch of kernel `kern`: `np` pages of the object starting at page
+// index `p0`.
+t2i_status noalloc_one(const NoAllocDevice& d, int kern, uint32_t k, const void* pool, int shift,
+                       const uint32_t* pages, uint64_t p0, uint64_t np, uint64_t nbytes, unsigned char* dst, bool cast,
+                       cudaStream_t stream) {
     thread_local LaunchParams<kBlobLarge> p;  // host-side parameter staging (no device memory)
     const uint64_t P = uint64_t(1) << shift;
     const uint64_t off = p0 * P;
@@ -1118,9 +1118,13 @@ t2i_status noalloc_one(const NoAllocDevice& d, uint32_t k, const void* pool, int
     std::memcpy(p.blob, &s, sizeof(s));
     std::memcpy(p.blob + sizeof(SegDesc), pages + p0, np * sizeof(uint32_t));
     const uint64_t want = (seg_bytes + kMinCtaBytes - 1) / kMinCtaBytes;
-    const unsigned grid =
-        static_cast<unsigned>(std::max<uint64_t>(1, std::min<uint64_t>(want, uint64_t(d.max_ctas[GENERAL ? 1 : 0]))));
-    cudaError_t e = noalloc_launch<GENERAL, kBlobLarge>(p, grid, stream);
+    const unsigned grid = static_cast<unsigned>(std::max<uint64_t>(1, std::min<uint64_t>(want, uint64_t(d.max_ctas[kern]))));
+    cudaLaunchConfig_t lc = {};
+    lc.gridDim = dim3(grid);
+    lc.blockDim = dim3(kThreads);
+    lc.stream = stream;
+    void* args[] = {&p};
+    cudaError_t e = cudaLaunchKernelExC(&lc, noalloc_kernel(kern), args);
     if (e != cudaSuccess) {
         set_thread_error(std::string("t2i_gather_noalloc: kernel launch failed: ") + cudaGetErrorString(e));
         return T2I_ERR_CUDA;
@@ -1208,15 +1212,12 @@ extern "C" t2i_status t2i_gather_noalloc(const void* pool_dev, uint64_t pool_byt
                              cudaGetErrorString(e));
             return T2I_ERR_CUDA;
         }
-        const bool general = (da & 15u) != 0;
+        const int kern = (da & 15u) == 0 ? kNoAllocGetAligned : cast ? kNoAllocGetAny : kNoAllocCopyAny;
         unsigned char* dst = static_cast<unsigned char*>(dst_dev);
         for (uint64_t k = 0; k < n_launch; ++k) {
             const uint64_t p0 = k * per_launch;
             const uint64_t np = std::min<uint64_t>(per_launch, n_pages - p0);
-            st = general ? noalloc_one<true>(*d, uint32_t(k), pool_dev, shift, pages, p0, np, nbytes, dst, cast != 0,
-                                             stream)
-                         : noalloc_one<false>(*d, uint32_t(k), pool_dev, shift, pages, p0, np, nbytes, dst,
-                                              cast != 0, stream);
+            st = noalloc_one(*d, kern, uint32_t(k), pool_dev, shift, pages, p0, np, nbytes, dst, cast != 0, stream);
             if (st != T2I_OK) return st;
         }
         return T2I_OK;

@@ -188,12 +188,13 @@ def test_object_larger_than_64_gib():
 
 
 def test_large_unaligned_launches_take_chunks():
-    """A 400 MiB object put from a source 3 bytes past alignment and got into
+    """A 704 MiB object put from a source 3 bytes past alignment and got into
     destinations 5 bytes (copy) and 2 bytes (cast) past it: launches large
-    enough for chunks from the work counter, in the any-alignment kernels."""
+    enough for chunks from the work counter (at least 1 MiB per resident
+    CTA of the any-alignment kernels, 4 per SM), in those kernels."""
     P = 2 << 20
-    n = 400 << 20
-    st = store(210 * P, P)
+    n = 704 << 20
+    st = store(360 * P, P)
     g = torch.Generator(device=DEV)
     g.manual_seed(400)
     f = torch.randn(n // 4, generator=g, device=DEV)

@@ -1,10 +1,15 @@
 """The allocation-free gather (t2i_gather_noalloc), called through the C ABI
-and compared with the store's own get (t2i_get_batch) on the same object
 (marked gpu). It serves callers that cannot allocate device memory while
 they move data, such as a serving process whose free HBM an inference engine
-or PyTorch's caching allocator has already reserved. Each case makes two
-calls in a row, because every call shares the library's static scratch
-counters and the second must not see what the first left behind.
+or PyTorch's caching allocator has already reserved.
+
+Every output is compared with what the oracle fixes for it: the object's own
+bytes (get(put(x)) == x), or, with the cast, the oracle's round-to-nearest-
+even of those bytes (oracle.cast, written independently of the kernels).
+Each case makes two calls in a row, because every call shares the library's
+static scratch counters and the second must not see what the first left
+behind. The cast inputs are random bit patterns, so NaNs, infinities,
+subnormals and exact ties all occur.
 
 This file is collected last on purpose: a failure here stops a first-failure
 run only after every other test has run."""
@@ -14,11 +19,13 @@ import numpy as np
 import pytest
 import torch
 
+from oracle.cast import f32_bits_to_bf16_bits
 from paper_2607_26566_gb300 import Store, _lib as L, get_descs, put_descs
 
 pytestmark = pytest.mark.gpu
 DEV = torch.device("cuda", 0)
 INVALID = 1
+GUARD = 64
 
 
 @pytest.fixture(scope="module", autouse=True)
@@ -45,60 +52,88 @@ def stored(P, pool_pages, x):
     return st, pool, int(i), st.ctl.object(int(i))[2]
 
 
-def reference(st, oid, n_out, cast, offset=0):
-    """The store's own get of the object into a fresh buffer."""
-    ref = torch.zeros(n_out + offset, dtype=torch.uint8, device=DEV)
-    s, _ = st.get_batch(get_descs([oid], [ref.data_ptr() + offset], dst_bytes=[n_out], cast=cast))
-    assert s == 0, st.last_error()
-    return ref
+def random_f32_bits(n_floats: int, seed: int) -> torch.Tensor:
+    """n_floats random fp32 bit patterns on the device, as bytes."""
+    g = np.random.default_rng(seed)
+    return torch.from_numpy(g.integers(0, 1 << 32, n_floats, dtype=np.uint64).astype(np.uint32)
+                            .view(np.uint8)).to(DEV)
+
+
+def expected(x: torch.Tensor, cast: int) -> np.ndarray:
+    """What the oracle fixes for the output: the bytes, or their RNE cast."""
+    raw = x.cpu().numpy()
+    return f32_bits_to_bf16_bits(raw.view(np.uint32)).view(np.uint8) if cast else raw
+
+
+def run_twice(pool, P, pages, x, cast, offset):
+    """Two calls in a row, each into a fresh buffer at `offset` bytes past a
+    256-byte boundary with guard bytes around it; returns the outputs."""
+    n_out = x.numel() // 2 if cast else x.numel()
+    outs = []
+    for _ in range(2):
+        buf = torch.full((n_out + offset + GUARD,), 0xA5, dtype=torch.uint8, device=DEV)
+        st = noalloc(pool, P, pages, x.numel(), buf.data_ptr() + offset, n_out, cast)
+        assert st == 0, L.load().t2i_last_error(None)
+        torch.cuda.synchronize()
+        h = buf.cpu().numpy()
+        assert (h[:offset] == 0xA5).all() and (h[offset + n_out:] == 0xA5).all(), "wrote outside the destination"
+        outs.append(h[offset:offset + n_out])
+    return outs
 
 
 @pytest.mark.parametrize("cast", [0, 1])
-def test_two_calls_match_get_batch(cast):
+def test_two_calls_match_the_oracle(cast):
     """fp32 object of 3 MiB + 12 bytes in 64 KiB pages (ragged last page),
-    copied or cast; two calls in a row into separate buffers."""
+    copied or cast into an aligned destination; the store's own get gives
+    the same bytes."""
     P = 64 * 1024
-    x = torch.randn((3 * (1 << 20) + 12) // 4, dtype=torch.float32, device=DEV).view(torch.uint8)
+    x = random_f32_bits((3 * (1 << 20) + 12) // 4, seed=1 + cast)
     st, pool, oid, pages = stored(P, 64, x)
-    n_out = x.numel() // 2 if cast else x.numel()
-    ref = reference(st, oid, n_out, cast)
-    outs = [torch.zeros(n_out, dtype=torch.uint8, device=DEV) for _ in range(2)]
-    for o in outs:
-        assert noalloc(pool, P, pages, x.numel(), o.data_ptr(), n_out, cast) == 0, L.load().t2i_last_error(None)
-    torch.cuda.synchronize()
-    for o in outs:
-        assert torch.equal(o, ref)
+    want = expected(x, cast)
+    for out in run_twice(pool, P, pages, x, cast, 0):
+        assert np.array_equal(out, want)
+    ref = torch.empty(want.size, dtype=torch.uint8, device=DEV)
+    s, _ = st.get_batch(get_descs([oid], [ref], cast=cast))
+    assert s == 0, st.last_error()
+    assert np.array_equal(ref.cpu().numpy(), want)
 
 
 def test_two_calls_multi_launch_unaligned():
-    """9,000 pages of 256 B (two launches, two scratch counters) into a
-    destination 3 bytes past 16-byte alignment (the any-alignment kernel)."""
+    """9,000 pages of 256 B (two launches, two scratch counters) copied into a
+    destination 3 bytes past 16-byte alignment (the any-alignment copy)."""
     P = 256
     x = torch.randint(0, 256, (9000 * P - 100,), dtype=torch.uint8, device=DEV)
     st, pool, oid, pages = stored(P, 9500, x)
     assert len(pages) == 9000
-    ref = reference(st, oid, x.numel(), 0, offset=3)
-    for _ in range(2):
-        out = torch.zeros_like(ref)
-        assert noalloc(pool, P, pages, x.numel(), out.data_ptr() + 3, x.numel(), 0) == 0, \
-            L.load().t2i_last_error(None)
-        torch.cuda.synchronize()
-        assert torch.equal(out, ref) and torch.equal(out[3:], x)
+    want = expected(x, 0)
+    for out in run_twice(pool, P, pages, x, 0, 3):
+        assert np.array_equal(out, want)
 
 
-def test_two_calls_large_object_cast():
-    """256 MiB of fp32 in 2 MiB pages: ~18 chunks per CTA, cast to bf16."""
+@pytest.mark.parametrize("offset", [2, 6, 14])
+def test_cast_into_2_byte_aligned_destination_two_launches(offset):
+    """An fp32 object of 9,000 pages of 256 B with a ragged last page (two
+    launches) cast into a destination that is 2-byte but not 16-byte
+    aligned (the any-alignment cast)."""
+    P = 256
+    x = random_f32_bits((9000 * P - 100) // 4, seed=10 + offset)
+    st, pool, oid, pages = stored(P, 9500, x)
+    assert len(pages) == 9000
+    want = expected(x, 1)
+    for out in run_twice(pool, P, pages, x, 1, offset):
+        assert np.array_equal(out, want)
+
+
+@pytest.mark.parametrize("offset", [0, 6])
+def test_two_calls_large_object_cast(offset):
+    """256 MiB of fp32 in 2 MiB pages (~18 chunks per CTA), cast to bf16
+    into an aligned destination and one 6 bytes past alignment."""
     P = 2 << 20
-    x = torch.randn(64 << 20, dtype=torch.float32, device=DEV).view(torch.uint8)
+    x = random_f32_bits(64 << 20, seed=20 + offset)
     st, pool, oid, pages = stored(P, 130, x)
-    n_out = x.numel() // 2
-    ref = reference(st, oid, n_out, 1)
-    for _ in range(2):
-        out = torch.zeros(n_out, dtype=torch.uint8, device=DEV)
-        assert noalloc(pool, P, pages, x.numel(), out.data_ptr(), n_out, 1) == 0, L.load().t2i_last_error(None)
-        torch.cuda.synchronize()
-        assert torch.equal(out, ref)
-    assert torch.equal(ref.view(torch.bfloat16), x.view(torch.float32).to(torch.bfloat16))
+    want = expected(x, 1)
+    for out in run_twice(pool, P, pages, x, 1, offset):
+        assert np.array_equal(out, want)
 
 
 def test_sizes_beyond_the_maximum_are_rejected():
