@@ -59,7 +59,7 @@ def parse():
     p.add_argument("--no-sweep", action="store_true", help="skip timing B = 1 and B = 4")
     p.add_argument("--pool-gib", type=float, default=None, help="smaller pool (profiling small cases)")
     p.add_argument("--cpu-seconds", type=float, default=10.0, help="minimum CPU-baseline sample time")
-    p.add_argument("--rows", default="tiny,weights,adapters,compaction,prefix,views,pull,host",
+    p.add_argument("--rows", default="tiny,unaligned,cdriver,weights,adapters,compaction,prefix,views,pull,host",
                    help="other hot-path rows timed in the same run (comma list, or 'none')")
     p.add_argument("--adapter-calls", type=int, default=10_000)
     p.add_argument("--adapter-sets", type=int, default=None, help="fewer LoRA sets (profiling small cases)")
@@ -209,6 +209,13 @@ class Handoff:
         self.ids_p = [C.cast(C.c_void_p(self.ids.ctypes.data + 8 * self.n_obj * r), C.POINTER(C.c_uint64))
                       for r in range(requests)]
         self.all_ids_p = self.ids.ctypes.data_as(C.POINTER(C.c_uint64))
+        # the CPython entry points (csrc/pycall.c) take plain integers: the
+        # same calls without ctypes' per-call conversion (None: ctypes only)
+        self.fast = L.pycall()
+        self.pd_a = [int(d.ctypes.data) for d in self.pd]
+        self.gd_a = [int(d.ctypes.data) for d in self.gd]
+        self.ids_a = [int(self.ids.ctypes.data) + 8 * self.n_obj * r for r in range(requests)]
+        self.hi = self.store._hi
         payload = sum(sp.nbytes for sp in self.specs)
         lat = self.specs[self.ci].nbytes
         self.put_bytes = 2 * payload * requests
@@ -221,27 +228,56 @@ class Handoff:
         """One step. ``ev`` = three events recorded before the puts, between
         the puts and the gets, and after the gets: each phase is a run of
         back-to-back launches of one kernel."""
-        lib, h, n = self.lib, self.h, self.n_obj
-        s = C.c_void_p(stream)
         if ev is not None:
             ev[0].record()
-        for r in range(self.requests):
-            st = lib.t2i_put_batch(h, self.pd_p[r], n, self.ids_p[r], s)
-            if st:
-                raise RuntimeError("put_batch: " + self.store.last_error())
+        self._puts([stream])
         if ev is not None:
             ev[1].record()
-        for r in range(self.requests):
-            self.gd[r]["id"] = self.ids[n * r:n * (r + 1)]
-            st = lib.t2i_get_batch(h, self.gd_p[r], n, None, s)
-            if st:
-                raise RuntimeError("get_batch: " + self.store.last_error())
+        self._gets([stream])
         if ev is not None:
             ev[2].record()
-        if not self.consumers:
-            st = lib.t2i_free(h, self.all_ids_p, len(self.ids))
-            if st:
-                raise RuntimeError("free: " + self.store.last_error())
+        self._free()
+
+    def _puts(self, streams):
+        """The put of every request, request r on ``streams[r % len]``
+        (cudaStream_t integers)."""
+        n, k, R = self.n_obj, len(streams), self.requests
+        if self.fast is not None:
+            put, hi, pd, ids = self.fast.put_batch, self.hi, self.pd_a, self.ids_a
+            for r in range(R):
+                if put(hi, pd[r], n, ids[r], streams[r % k]):
+                    raise RuntimeError("put_batch: " + self.store.last_error())
+            return
+        lib, h = self.lib, self.h
+        ss = [C.c_void_p(x) for x in streams]
+        for r in range(R):
+            if lib.t2i_put_batch(h, self.pd_p[r], n, self.ids_p[r], ss[r % k]):
+                raise RuntimeError("put_batch: " + self.store.last_error())
+
+    def _gets(self, streams):
+        """The get of every request (with the ids of its put), request r on
+        ``streams[r % len]``."""
+        n, k, R = self.n_obj, len(streams), self.requests
+        if self.fast is not None:
+            get, hi, gd, ids = self.fast.get_batch_ids, self.hi, self.gd_a, self.ids_a
+            for r in range(R):
+                if get(hi, gd[r], n, ids[r], 0, streams[r % k]):
+                    raise RuntimeError("get_batch: " + self.store.last_error())
+            return
+        lib, h = self.lib, self.h
+        ss = [C.c_void_p(x) for x in streams]
+        for r in range(R):
+            self.gd[r]["id"] = self.ids[n * r:n * (r + 1)]
+            if lib.t2i_get_batch(h, self.gd_p[r], n, None, ss[r % k]):
+                raise RuntimeError("get_batch: " + self.store.last_error())
+
+    def _free(self):
+        if self.consumers:
+            return
+        st = (self.fast.free(self.hi, int(self.ids.ctypes.data), len(self.ids)) if self.fast is not None
+              else self.lib.t2i_free(self.h, self.all_ids_p, len(self.ids)))
+        if st:
+            raise RuntimeError("free: " + self.store.last_error())
 
     def step_streams(self, streams, ev=None):
         """One step with request r on ``streams[r % k]``: independent requests
@@ -251,25 +287,14 @@ class Handoff:
         events), so no further synchronisation is needed; the two phases
         are still joined through ``streams[0]`` so that each phase's span is
         measurable. ``ev`` = three timing events as in :meth:`step`."""
-        lib, h, n, k = self.lib, self.h, self.n_obj, len(streams)
-        ss = [C.c_void_p(x.cuda_stream) for x in streams]
+        ss = [int(x.cuda_stream) for x in streams]
         if ev is not None:
             ev[0].record(streams[0])
-        for r in range(self.requests):
-            st = lib.t2i_put_batch(h, self.pd_p[r], n, self.ids_p[r], ss[r % k])
-            if st:
-                raise RuntimeError("put_batch: " + self.store.last_error())
+        self._puts(ss)
         self._join(streams, ev[1] if ev is not None else None)
-        for r in range(self.requests):
-            self.gd[r]["id"] = self.ids[n * r:n * (r + 1)]
-            st = lib.t2i_get_batch(h, self.gd_p[r], n, None, ss[r % k])
-            if st:
-                raise RuntimeError("get_batch: " + self.store.last_error())
+        self._gets(ss)
         self._join(streams, ev[2] if ev is not None else None)
-        if not self.consumers:
-            st = lib.t2i_free(h, self.all_ids_p, len(self.ids))
-            if st:
-                raise RuntimeError("free: " + self.store.last_error())
+        self._free()
 
     def _join(self, streams, hub_event=None):
         """Every stream waits until all of them reach this point (through
@@ -291,20 +316,24 @@ class Handoff:
         store orders each get after the put of its request only, so request
         r+1's put overlaps request r's get (both directions of the host link
         in the end-to-end case)."""
-        lib, h, n = self.lib, self.h, self.n_obj
-        sp, sg = C.c_void_p(s_put.cuda_stream), C.c_void_p(s_get.cuda_stream)
-        for r in range(self.requests):
-            st = lib.t2i_put_batch(h, self.pd_p[r], n, self.ids_p[r], sp)
-            if st:
-                raise RuntimeError("put_batch: " + self.store.last_error())
-            self.gd[r]["id"] = self.ids[n * r:n * (r + 1)]
-            st = lib.t2i_get_batch(h, self.gd_p[r], n, None, sg)
-            if st:
-                raise RuntimeError("get_batch: " + self.store.last_error())
-        if not self.consumers:
-            st = lib.t2i_free(h, self.all_ids_p, len(self.ids))
-            if st:
-                raise RuntimeError("free: " + self.store.last_error())
+        n = self.n_obj
+        sp, sg = int(s_put.cuda_stream), int(s_get.cuda_stream)
+        if self.fast is not None:
+            put, get, hi = self.fast.put_batch, self.fast.get_batch_ids, self.hi
+            for r in range(self.requests):
+                if put(hi, self.pd_a[r], n, self.ids_a[r], sp):
+                    raise RuntimeError("put_batch: " + self.store.last_error())
+                if get(hi, self.gd_a[r], n, self.ids_a[r], 0, sg):
+                    raise RuntimeError("get_batch: " + self.store.last_error())
+        else:
+            lib, h = self.lib, self.h
+            for r in range(self.requests):
+                if lib.t2i_put_batch(h, self.pd_p[r], n, self.ids_p[r], C.c_void_p(sp)):
+                    raise RuntimeError("put_batch: " + self.store.last_error())
+                self.gd[r]["id"] = self.ids[n * r:n * (r + 1)]
+                if lib.t2i_get_batch(h, self.gd_p[r], n, None, C.c_void_p(sg)):
+                    raise RuntimeError("get_batch: " + self.store.last_error())
+        self._free()
 
     def step_one_call(self):
         """The same step with one put_batch of all requests' objects and one
@@ -333,6 +362,7 @@ class Handoff:
                            d2h_mode=d2h_mode)
         self.lib = self.store._lib
         self.h = self.store._h
+        self.hi = self.store._hi
 
     def verify(self):
         """get(put(x)) == x on every output after a step: byte equality, and
@@ -571,6 +601,96 @@ def time_tiny(device, reps: int = 20):
     return {"workload": "tiny: 64 MiB pool, 64 KiB pages, 32 + 8 uint8 objects (1 KiB - 2 MiB)",
             "ms_per_step": round(ms, 4), "gbs": round(payload / (ms * 1e-3) / 1e9, 1), "bit_exact": bool(ok),
             "launches_per_step": 4}
+
+
+def time_unaligned(device, reps: int = 10, nbytes: int = 1 << 30):
+    """The any-alignment kernels on one 1 GiB object (2 MiB pages, a 2 GiB
+    pool): puts from sources 1, 4 and 8 bytes past a 16-byte boundary, gets
+    into destinations 1 and 3 bytes past one, fp32 -> bf16 casts into
+    destinations 2 and 6 bytes past one, each beside its aligned form. Every
+    call is timed alone with CUDA events (median of ``reps``); the outputs of
+    the last calls are compared with the input (the casts with torch's own
+    round-to-nearest-even conversion)."""
+    import torch
+
+    from paper_2607_26566_gb300 import Store, get_descs, put_descs
+
+    stream = torch.cuda.current_stream(device)
+    src = torch.randn(nbytes // 4 + 16, dtype=torch.float32, device=device).view(torch.uint8)
+    dst = torch.empty(nbytes + 64, dtype=torch.uint8, device=device)
+    pool = torch.empty(2 << 30, dtype=torch.uint8, device=device)
+    st = Store(pool, 2 << 20)
+    ev = [torch.cuda.Event(enable_timing=True) for _ in range(2)]
+
+    def timed(fn):
+        ms = []
+        for _ in range(reps + 2):
+            ev[0].record(stream)
+            fn()
+            ev[1].record(stream)
+            torch.cuda.synchronize(device)
+            ms.append(ev[0].elapsed_time(ev[1]))
+        return statistics.median(ms[2:])
+
+    out = {"workload": "one 1 GiB object, 2 MiB pages, user addresses at byte offsets from a 16-byte boundary",
+           "reps": reps}
+    ids = [0]
+
+    def put(off):
+        def fn():
+            if ids[0]:
+                st.check(st.free([ids[0]]))
+            s, got = st.put_batch(put_descs([src.data_ptr() + off], nbytes=[nbytes]))
+            st.check(s)
+            ids[0] = int(got[0])
+        return fn
+
+    for off in (0, 1, 4, 8):
+        out[f"put_src+{off}_gbs"] = round(2 * nbytes / (timed(put(off)) * 1e-3) / 1e9, 1)
+    put(0)()  # the object now holds src[:nbytes], which the gets read back
+
+    def get(off, cast):
+        n_out = nbytes // 2 if cast else nbytes
+        d = get_descs([ids[0]], [dst.data_ptr() + off], dst_bytes=[n_out], cast=cast)
+        return lambda: st.check(st.get_batch(d, per_item=False)[0])
+
+    for off in (0, 1, 3):
+        out[f"get_dst+{off}_gbs"] = round(2 * nbytes / (timed(get(off, 0)) * 1e-3) / 1e9, 1)
+    ok = torch.equal(dst[3:3 + nbytes], src[:nbytes])
+    for off in (0, 2, 6):
+        out[f"cast_dst+{off}_gbs"] = round(1.5 * nbytes / (timed(get(off, 1)) * 1e-3) / 1e9, 1)
+    want = src[:nbytes].view(torch.float32).to(torch.bfloat16).view(torch.uint8)
+    ok = ok and torch.equal(dst[6:6 + nbytes // 2], want)
+    put(1)()
+    get(1, 0)()
+    torch.cuda.synchronize(device)
+    ok = ok and torch.equal(dst[1:1 + nbytes], src[1:1 + nbytes])
+    out["bit_exact"] = bool(ok)
+    st.close()
+    return out
+
+
+def time_c_driver(steps: int = 50, warmup: int = 3):
+    """The handoff step driven from C through the C ABI (cdriver/handoff_step.c,
+    no Python between calls), 64 requests of 2 MiB pages in an 8 GiB pool:
+    B = 1 and 8, on 4 streams and on one. Its host microseconds per call are
+    the library's own cost (pointer checks, directory, page dependencies,
+    launch); the gap to the Python rows is the binding's."""
+    from paper_2607_26566_gb300 import build as b
+
+    exe = b.build_cdriver()
+    out = {"workload": "t2i handoff, 64 requests, 2 MiB pages, 8 GiB pool, driven from C", "runs": []}
+    for B, S in ((1, 4), (1, 1), (8, 4), (8, 1)):
+        r = subprocess.run([exe, str(B), "64", str(S), str(steps), str(warmup)], capture_output=True, text=True,
+                           timeout=600)
+        if r.returncode:
+            raise RuntimeError(f"C driver B={B} S={S} failed: {r.stderr.strip()[-400:]}")
+        d = json.loads(r.stdout.strip().splitlines()[-1])
+        if not d["outputs_ok"]:
+            raise RuntimeError(f"C driver B={B} S={S}: an output differs from its input")
+        out["runs"].append({k: d[k] for k in ("B", "streams", "gbs", "ms_per_step", "host_us_per_put",
+                                              "host_us_per_get")})
+    return out
 
 
 # ----------------------------------------------------------------------------- weights
@@ -1752,6 +1872,10 @@ def run_rows(args, device, peak):
     wanted = [] if args.rows == "none" else [r.strip() for r in args.rows.split(",") if r.strip()]
     if "tiny" in wanted:
         rows["tiny"] = time_tiny(device)
+    if "unaligned" in wanted:
+        rows["unaligned"] = time_unaligned(device)
+    if "cdriver" in wanted:
+        rows["cdriver"] = time_c_driver()
     if "host" in wanted:
         rows["host"] = time_host_control()
     if "weights" in wanted:

@@ -101,6 +101,7 @@ PROTOTYPES = {
 }
 
 _lib = None
+_pycall = False  # not looked up yet
 
 
 def load() -> C.CDLL:
@@ -117,3 +118,19 @@ def load() -> C.CDLL:
             fn.argtypes = args
         _lib = lib
     return _lib
+
+
+def pycall():
+    """The CPython entry points of csrc/pycall.c (put_batch, get_batch,
+    get_batch_ids, free: the same C-ABI calls without ctypes' per-call
+    argument conversion), or None where Python.h was missing at build time.
+    Loads the library first."""
+    global _pycall
+    if _pycall is False:
+        load()
+        try:
+            from . import _pycall as m
+        except ImportError:
+            m = None
+        _pycall = m
+    return _pycall

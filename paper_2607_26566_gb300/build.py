@@ -12,6 +12,7 @@ import os
 import shutil
 import subprocess
 import sys
+import sysconfig
 
 PKG = os.path.dirname(os.path.abspath(__file__))
 ROOT = os.path.dirname(PKG)
@@ -19,6 +20,10 @@ CSRC = os.path.join(PKG, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(PKG, "libt2istore.so")
+# CPython entry points for the per-request calls (csrc/pycall.c), linked
+# against LIB
+PYCALL_SRC = "pycall.c"
+PYCALL = os.path.join(PKG, "_pycall" + (sysconfig.get_config_var("EXT_SUFFIX") or ".so"))
 
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 CXX_SOURCES = ["control.cpp", "ctl_capi.cpp", "prefix.cpp"]
@@ -36,7 +41,7 @@ def _cuda_home() -> str:
 
 
 def _inputs() -> list[str]:
-    files = [os.path.join(CSRC, f) for f in CXX_SOURCES + CU_SOURCES + HEADERS]
+    files = [os.path.join(CSRC, f) for f in CXX_SOURCES + CU_SOURCES + HEADERS + [PYCALL_SRC]]
     return files + [os.path.join(INCLUDE, "t2istore.h"), os.path.abspath(__file__)]
 
 
@@ -52,10 +57,15 @@ def kernel_source_hash() -> str:
     return h.hexdigest()[:12]
 
 
+def _have_python_h() -> bool:
+    return os.path.exists(os.path.join(sysconfig.get_paths()["include"], "Python.h"))
+
+
 def is_stale() -> bool:
-    if not os.path.exists(LIB):
+    outs = [LIB] + ([PYCALL] if _have_python_h() else [])
+    if not all(os.path.exists(f) for f in outs):
         return True
-    t = os.path.getmtime(LIB)
+    t = min(os.path.getmtime(f) for f in outs)
     return any(os.path.getmtime(f) > t for f in _inputs())
 
 
@@ -87,9 +97,9 @@ def build(verbose: bool = False, ptxas_info: bool = False, defines=(), out: str 
     objs = []
     errors = []
     for p, cmd, obj in procs:
-        out, _ = p.communicate()
+        log, _ = p.communicate()
         if verbose or ptxas_info or p.returncode:
-            sys.stderr.write(out)
+            sys.stderr.write(log)
         if p.returncode:
             errors.append(" ".join(cmd))
         objs.append(obj)
@@ -104,7 +114,48 @@ def build(verbose: bool = False, ptxas_info: bool = False, defines=(), out: str 
     if r.returncode:
         raise RuntimeError("link failed: " + " ".join(link))
     os.replace(tmp, lib_path)
+    if out is None:
+        if _have_python_h():
+            build_pycall(verbose)
+        else:
+            # the ctypes binding serves every call; only its per-call cost is higher
+            sys.stderr.write("build: Python.h not found; the CPython binding (_pycall) is not built\n")
     return lib_path
+
+
+def build_pycall(verbose: bool = False) -> str:
+    """Compiles the CPython module of csrc/pycall.c next to LIB (linked
+    against it, found through $ORIGIN). Raises on failure."""
+    py_inc = sysconfig.get_paths()["include"]
+    if not os.path.exists(os.path.join(py_inc, "Python.h")):
+        raise RuntimeError(f"Python.h not found in {py_inc}: the CPython binding cannot be built")
+    tmp = PYCALL + ".tmp"
+    cmd = [os.environ.get("CC", "gcc"), "-O2", "-shared", "-fPIC", "-Wall", os.path.join(CSRC, PYCALL_SRC),
+           "-I" + INCLUDE, "-I" + py_inc, "-L" + PKG, "-lt2istore", "-Wl,-rpath,$ORIGIN", "-o", tmp]
+    r = subprocess.run(cmd, stdout=subprocess.PIPE, stderr=subprocess.STDOUT, text=True)
+    if verbose or r.returncode:
+        sys.stderr.write(r.stdout)
+    if r.returncode:
+        raise RuntimeError("CPython binding build failed: " + " ".join(cmd))
+    os.replace(tmp, PYCALL)
+    return PYCALL
+
+
+def build_cdriver() -> str:
+    """Compiles cdriver/handoff_step.c (the handoff workload driven from C
+    through the C ABI) into _build/ against LIB and the CUDA runtime;
+    returns the executable's path. Raises on failure."""
+    cuda = _cuda_home()
+    os.makedirs(BUILD, exist_ok=True)
+    exe = os.path.join(BUILD, "handoff_step")
+    lib64 = os.path.join(cuda, "lib64")
+    cmd = [os.environ.get("CC", "gcc"), "-O2", "-std=c11", "-Wall", os.path.join(PKG, "cdriver", "handoff_step.c"),
+           "-I" + INCLUDE, "-I" + os.path.join(cuda, "include"), "-L" + PKG, "-lt2istore", "-L" + lib64, "-lcudart",
+           "-Wl,-rpath," + PKG + ":" + lib64, "-o", exe]
+    r = subprocess.run(cmd, stdout=subprocess.PIPE, stderr=subprocess.STDOUT, text=True)
+    if r.returncode:
+        raise RuntimeError("C driver build failed: " + " ".join(cmd) + "\n" + r.stdout)
+    return exe
 
 
 def ensure_built() -> str:

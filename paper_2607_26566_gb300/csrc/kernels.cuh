@@ -113,9 +113,18 @@ struct LaunchHeader {
     uint32_t piece_bytes;     // min(U, page size)
     uint32_t pages_offset;    // byte offset of the uint32 page array in blob
     uint32_t chunk_granules;  // granules a CTA takes at a time from the counter
-    uint32_t pad[2];
+    uint32_t flags;           // kPrefetchSources, or 0
+    uint32_t prefetch_ctas;   // CTAs 0 .. prefetch_ctas-1 prefetch their shares (kPrefetchSources)
 };
 static_assert(sizeof(LaunchHeader) == 48, "LaunchHeader layout");
+// Every source byte of the launch is device memory: a CTA with an equal
+// static share may ask L2 for its source bytes before the previous grid on
+// the stream has completed (prefetch_share).
+constexpr uint32_t kPrefetchSources = 1u;
+#ifndef T2I_TUNE_PREFETCH
+#define T2I_TUNE_PREFETCH 1
+#endif
+constexpr bool kPrefetch = T2I_TUNE_PREFETCH != 0;
 
 // The chunk counter of one stream of a store. Zero between launches: the
 // last CTA of every launch that used it puts both fields back to zero, and
@@ -453,6 +462,66 @@ __device__ __forceinline__ uint32_t find_segment(const SegDesc* segs, uint32_t n
     return lo;
 }
 
+// Asks L2 for the first source bytes of this CTA's equal static share (the
+// first contiguous source range, at most kPrefetchMax bytes), one 128-byte
+// line per thread, before the CTA waits for the previous grid on the stream.
+// A CTA of the next launch becomes resident as soon as a CTA of the draining
+// one exits, so its first HBM reads overlap that drain instead of following
+// it. A prefetch is only a cache hint: it changes no value that a load
+// returns (L2 serves every SM's loads), so a source that the previous grid
+// is still writing is read correctly after the wait. Sources are device
+// memory (the host sets kPrefetchSources only then), and every line holds a
+// source byte, so no prefetch leaves the source allocation.
+// A sweep on GB300 (handoff B=8 request per launch; 256-object adapter
+// gets): one round (32 KiB) by every CTA lifted one-stream puts by 2.8%,
+// one-stream gets by 3.5% and adapter gets by 2.1%, and left the 4-stream
+// handoff unchanged (+0.1%); the whole 64 KiB share cost the 4-stream put
+// 2.2% and adapter gets 2%, and prefetching in the first wave of CTAs only
+// gained less. A single bulk prefetch (cp.async.bulk.prefetch) per range
+// cost the copy loop ~200 bytes of register spills, so the lines are
+// prefetched one per thread.
+#ifndef T2I_TUNE_PREFETCH_BYTES
+#define T2I_TUNE_PREFETCH_BYTES (32 * 1024)
+#endif
+#ifndef T2I_TUNE_PREFETCH_WAVE
+#define T2I_TUNE_PREFETCH_WAVE 0
+#endif
+constexpr uint64_t kPrefetchMax = T2I_TUNE_PREFETCH_BYTES;
+// 1: only the first wave of CTAs (those resident at launch) prefetches
+constexpr bool kPrefetchFirstWave = T2I_TUNE_PREFETCH_WAVE != 0;
+
+template <Mode M, int BLOB>
+__device__ __forceinline__ void prefetch_share(const LaunchParams<BLOB>& p) {
+    if (!kPrefetch || p.h.work != 0 || !(p.h.flags & kPrefetchSources) || blockIdx.x >= p.h.prefetch_ctas) return;
+    constexpr bool kFromPool = M == Mode::Get || M == Mode::GetCopy;  // else the user address is the source
+    const SegDesc* segs = reinterpret_cast<const SegDesc*>(p.blob);
+    const uint32_t* pages = reinterpret_cast<const uint32_t*>(p.blob + p.h.pages_offset);
+    const uint32_t pshift = p.h.page_shift;
+    const uint64_t pmask = (uint64_t(1) << pshift) - 1;
+    const uint64_t g0 = uint64_t(p.h.n_granules) * blockIdx.x / gridDim.x;
+    const uint64_t g1 = uint64_t(p.h.n_granules) * (blockIdx.x + 1) / gridDim.x;
+    const SegDesc s = segs[find_segment(segs, p.h.n_seg, uint32_t(g0))];
+    const uint64_t off = g0 * kGranule - uint64_t(s.start) * kGranule;
+    const uint64_t nbytes = s.nbytes_flags & kSegBytesMask;
+    if (g0 == g1 || off >= nbytes) return;
+    uint64_t len = umin64(umin64((g1 - g0) * kGranule, nbytes - off), kPrefetchMax);
+    uint64_t a;
+    if (!kFromPool) {
+        a = s.user + off;
+    } else if (s.nbytes_flags & kRunFlag) {
+        a = p.h.pool + (uint64_t(pages[s.page_begin]) << pshift) + off;
+    } else {
+        len = umin64(len, pmask + 1 - (off & pmask));
+        a = p.h.pool + (uint64_t(pages[s.page_begin + (off >> pshift)]) << pshift) + (off & pmask);
+    }
+    // lines [a & ~127, a + len): each holds at least one source byte
+    const uint64_t first = a & ~uint64_t(127);
+    const uint32_t n_lines = uint32_t((a + len - first + 127) >> 7);
+#pragma unroll 1
+    for (uint32_t k = threadIdx.x; k < n_lines; k += kThreads)
+        asm volatile("prefetch.global.L2 [%0];" ::"l"(first + (uint64_t(k) << 7)));
+}
+
 // Programmatic dependent launch: wait until the previous grid in the stream
 // has completed and its memory is visible (returns at once when this launch
 // has no such dependency), then let the next launch begin its set-up.
@@ -593,12 +662,14 @@ __device__ __forceinline__ void run_range(const LaunchParams<BLOB>& p, uint64_t 
 template <int BLOB, bool GENERAL>
 __global__ void __launch_bounds__(kThreads, GENERAL ? kMinBlocksGeneral : kMinBlocks)
     scatter_put_kernel(const __grid_constant__ LaunchParams<BLOB> p) {
+    prefetch_share<Mode::Put, BLOB>(p);
     pdl_wait_then_release();
     run_share<Mode::Put, GENERAL, BLOB>(p);
 }
 template <int BLOB, bool GENERAL>
 __global__ void __launch_bounds__(kThreads, GENERAL ? kMinBlocksGeneralGet : kMinBlocksGet)
     gather_get_kernel(const __grid_constant__ LaunchParams<BLOB> p) {
+    prefetch_share<Mode::Get, BLOB>(p);
     pdl_wait_then_release();
     run_share<Mode::Get, GENERAL, BLOB>(p);
 }
@@ -607,11 +678,13 @@ __global__ void __launch_bounds__(kThreads, GENERAL ? kMinBlocksGeneralGet : kMi
 template <int BLOB, bool GENERAL>
 __global__ void __launch_bounds__(kThreads, GENERAL ? kMinBlocksGeneral : kMinBlocks)
     gather_copy_kernel(const __grid_constant__ LaunchParams<BLOB> p) {
+    prefetch_share<Mode::GetCopy, BLOB>(p);
     pdl_wait_then_release();
     run_share<Mode::GetCopy, GENERAL, BLOB>(p);
 }
 template <int BLOB>
 __global__ void __launch_bounds__(kThreads, kMinBlocks) compact_move_kernel(const __grid_constant__ LaunchParams<BLOB> p) {
+    prefetch_share<Mode::Move, BLOB>(p);
     pdl_wait_then_release();
     run_share<Mode::Move, false, BLOB>(p);
 }

@@ -28,7 +28,7 @@ t2i_status Store::launch_one(const std::vector<SegDesc>& sd, const std::vector<u
     p->h.pool = pool_;
     p->h.work = chunked ? cur_work_ : 0;
     p->h.chunk_granules = kChunkGranules;
-    p->h.pad[0] = p->h.pad[1] = 0;
+    p->h.flags = p->h.work == 0 ? launch_flags_ : 0;
     p->h.n_seg = static_cast<uint32_t>(sd.size());
     p->h.n_granules = n_granules;
     p->h.page_shift = page_shift_;
@@ -48,6 +48,7 @@ t2i_status Store::launch_one(const std::vector<SegDesc>& sd, const std::vector<u
     if (p->h.work == 0) g = std::max<uint64_t>(g, std::min<uint64_t>((bytes + kStaticCtaBytes - 1) / kStaticCtaBytes,
                                                                      0x7FFFFFFFull));
     const unsigned grid = static_cast<unsigned>(g);
+    p->h.prefetch_ctas = kPrefetchFirstWave ? static_cast<uint32_t>(std::min<uint64_t>(g, resident)) : grid;
     void* args[] = {p};
     const void* fn = M == Mode::Put                  ? reinterpret_cast<const void*>(scatter_put_kernel<BLOB, GENERAL>)
                      : mode == int(Mode::GetCopy)     ? reinterpret_cast<const void*>(gather_copy_kernel<BLOB, GENERAL>)

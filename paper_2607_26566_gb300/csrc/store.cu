@@ -243,6 +243,9 @@ class Store {
     static constexpr uint32_t kWorkStreams = 64;
     WorkCounter* work_ = nullptr;
     uint64_t cur_work_ = 0;  // the current call's counter (0: static shares)
+    // LaunchHeader::flags of the current call's launches with static
+    // shares: kPrefetchSources unless a put reads host or managed memory
+    uint32_t launch_flags_ = kPrefetchSources;
     std::vector<Seg> aligned_, general_;
     StreamDeps deps_;
     std::string err_;
@@ -336,6 +339,7 @@ t2i_status Store::put(const t2i_put_desc* descs, uint32_t n, t2i_id* ids, cudaSt
     std::vector<uint64_t> dev_src(n);
     std::vector<uint8_t> use_ce(n);
     Range cache;
+    bool device_sources = true;  // every source the kernel reads is device memory
     for (uint32_t i = 0; i < n; ++i) {
         const t2i_put_desc& d = descs[i];
         if (d.src_is_host > 1 || d.evictable > 1) {
@@ -349,6 +353,9 @@ t2i_status Store::put(const t2i_put_desc* descs, uint32_t n, t2i_id* ids, cudaSt
                 err_ = "put: item " + std::to_string(i) + ": " + err_;
                 return st;
             }
+            if (!ce && d.nbytes)
+                device_sources = device_sources && !d.src_is_host &&
+                                 (!cfg_.check_pointers || cache.kind == MemKind::Device);
         }
         use_ce[i] = ce;
     }
@@ -419,7 +426,9 @@ t2i_status Store::put(const t2i_put_desc* descs, uint32_t n, t2i_id* ids, cudaSt
         }
     }
     if (!segs_.empty()) {
+        launch_flags_ = device_sources ? kPrefetchSources : 0;
         st = launch_segments<Mode::Put>(segs_, stream);
+        launch_flags_ = kPrefetchSources;
         if (st != T2I_OK) {
             mark_writes();
             ctl_.rollback_put(ids, n);
@@ -1109,7 +1118,8 @@ t2i_status noalloc_one(const NoAllocDevice& d, int kern, uint32_t k, const void*
     p.h.piece_bytes = static_cast<uint32_t>(std::min<uint64_t>(kPieceBytes, P));
     p.h.pages_offset = sizeof(SegDesc);
     p.h.chunk_granules = kChunkGranules;
-    p.h.pad[0] = p.h.pad[1] = 0;
+    p.h.flags = 0;
+    p.h.prefetch_ctas = 0;
     SegDesc s;
     s.user = reinterpret_cast<uint64_t>(dst) + (cast ? off / 2 : off);
     s.nbytes_flags = seg_bytes | (cast ? kCastFlag : 0);

@@ -232,12 +232,15 @@ class Store:
         if st != L.OK:
             raise T2IError(st, self._lib.t2i_last_error(None).decode())
         self._h = h
+        self._hi = int(h.value)  # the handle as an integer, for the CPython entry points
+        self._fast = L.pycall()
         self.ctl = Ctl(_borrowed=self._lib.t2i_store_ctl(h), _owner=self)
 
     def close(self):
         if getattr(self, "_h", None):
             self._lib.t2i_store_destroy(self._h)
             self._h = None
+            self._hi = 0
 
     __del__ = close
 
@@ -270,6 +273,8 @@ class Store:
     def put_prepared(self, p: "Store.Prepared", stream=None):
         """(status, ids) -- t2i_put_batch on a prepared batch. ``ids`` is the
         batch's own array, overwritten by the next call."""
+        if self._fast is not None:
+            return self._fast.put_batch(self._hi, p.addr, p.n, p.out_addr, _stream(stream)), p.out
         return self._lib.t2i_put_batch(self._h, p.addr, p.n, p.out_addr, _stream(stream)), p.out
 
     def prepare_get(self, descs: np.ndarray) -> "Store.Prepared":
@@ -278,7 +283,13 @@ class Store:
 
     def get_prepared(self, p: "Store.Prepared", ids=None, stream=None) -> int:
         """t2i_get_batch on a prepared batch, after setting its ids to ``ids``
-        (if given); per-item statuses land in ``p.out``."""
+        (if given: a uint64 array of at least ``p.n`` ids, e.g. the ids a
+        prepared put returned); per-item statuses land in ``p.out``."""
+        if self._fast is not None and (ids is None or (isinstance(ids, np.ndarray) and ids.dtype == np.uint64
+                                                       and ids.flags.c_contiguous and len(ids) >= p.n)):
+            if ids is None:
+                return self._fast.get_batch(self._hi, p.addr, p.n, p.out_addr, _stream(stream))
+            return self._fast.get_batch_ids(self._hi, p.addr, p.n, ids.ctypes.data, p.out_addr, _stream(stream))
         if ids is not None:
             p.descs["id"] = ids
         return self._lib.t2i_get_batch(self._h, p.addr, p.n, p.out_addr, _stream(stream))

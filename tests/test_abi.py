@@ -208,3 +208,42 @@ def test_control_core_from_c_follows_the_hand_trace(lib, tmp_path):
                     str(exe), "-L" + lib_dir, "-l:libt2istore.so", "-Wl,-rpath," + lib_dir], check=True)
     out = subprocess.run([str(exe)], capture_output=True, text=True, check=True).stdout
     assert out == C_DRIVER_WANT
+
+
+def test_cpython_binding_marshals_only(lib):
+    """The CPython entry points pass their integer arguments to the same C-ABI
+    calls: a null store handle comes back INVALID from the library, the ids
+    given to get_batch_ids land in the descriptors' id fields first, and bad
+    argument lists raise before any call."""
+    import numpy as np
+
+    from paper_2607_26566_gb300 import build as b
+    from paper_2607_26566_gb300.store import GET_DTYPE
+
+    fast = L.pycall()
+    if fast is None:
+        assert not b._have_python_h()
+        pytest.skip("built without Python.h: the ctypes binding serves every call")
+    assert fast.put_batch(0, 0, 0, 0, 0) == L.ERR_INVALID
+    assert fast.get_batch(0, 0, 0, 0, 0) == L.ERR_INVALID
+    assert fast.free(0, 0, 0) == L.ERR_INVALID
+    descs = np.zeros(3, GET_DTYPE)
+    ids = np.array([7, 9, 11], np.uint64)
+    assert fast.get_batch_ids(0, descs.ctypes.data, 3, ids.ctypes.data, 0, 0) == L.ERR_INVALID
+    assert list(descs["id"]) == [7, 9, 11]
+    with pytest.raises(TypeError):
+        fast.put_batch(0, 0, 0, 0)
+    with pytest.raises(ValueError):
+        fast.get_batch_ids(0, 0, 2, 0, 0, 0)
+    with pytest.raises(OverflowError):
+        fast.get_batch(0, 0, 1 << 40, 0, 0)
+
+
+def test_c_driver_builds_against_the_header_and_library(lib):
+    """cdriver/handoff_step.c, the handoff workload driven from C through the
+    C ABI, compiles and links against include/t2istore.h and the library (it
+    runs in the GPU tests and the benchmark)."""
+    from paper_2607_26566_gb300 import build as b
+
+    exe = b.build_cdriver()
+    assert os.access(exe, os.X_OK)
