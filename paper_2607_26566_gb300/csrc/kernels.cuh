@@ -87,6 +87,12 @@ constexpr uint64_t kStaticCtaBytes = T2I_TUNE_STATIC_CTA_BYTES;
 #define T2I_TUNE_GET_COPY_KERNEL 1
 #endif
 constexpr bool kGetCopyKernel = T2I_TUNE_GET_COPY_KERNEL != 0;  // gets without casts run gather_copy_kernel
+#ifndef T2I_TUNE_CAST_SHUFFLE
+#define T2I_TUNE_CAST_SHUFFLE 1  // casts into unaligned destinations realign by warp shuffles (0: in shared memory)
+#endif
+#ifndef T2I_TUNE_CAST_SHUFFLE_STEPS
+#define T2I_TUNE_CAST_SHUFFLE_STEPS 5  // blocks of 8 floats in flight per thread in that cast
+#endif
 
 // One object segment of a launch. For a put/move the user address is the
 // source; for a get it is the destination. Bit 63 of nbytes_flags asks for
@@ -448,6 +454,94 @@ __device__ __noinline__ void cta_cast_staged(unsigned char* __restrict__ dst, co
     __syncthreads();  // the stage is free for the next piece
 }
 
+// fp32 (pool, 16-byte aligned) -> bf16 into a destination 2, 4, ..., 14
+// bytes past a 16-byte boundary, len <= U source bytes (a multiple of 4),
+// without shared memory. With h (1..7) elements before the destination's
+// first 16-byte boundary, aligned output vector k holds elements
+// [h + 8k, h + 8k + 8): the last 8 - h elements of source block k (floats
+// 8k .. 8k + 7) and the first h of block k + 1. Lane l of a warp loads and
+// casts block 31q + l, takes block 31q + l + 1 from lane l + 1 by a
+// shuffle, and lanes 0..30 store output vector 31q + l (the 32nd block is
+// loaded again by the next step: 1/31 more L2 reads, no more DRAM traffic).
+// The thread of block 0 also stores the h head elements, and the thread of
+// vector n8 (one past the last whole vector) the last < 8 elements, so
+// every load of a piece is issued before its first store. S steps of loads
+// per thread cover a whole piece in one round (8 warps x S x 31 vectors).
+// Source vectors past the piece's bytes are not read (each loaded vector
+// holds a source byte; a partial last vector lies in the same page).
+template <int Q, int S>
+__device__ __forceinline__ void emit_cast_shuffled(unsigned char* __restrict__ dst, const uint4* __restrict__ s,
+                                                   uint32_t h, uint32_t n8, uint32_t tail, uint32_t nvs,
+                                                   uint32_t r) {
+    constexpr uint32_t kWarps = kThreads / 32;
+    const uint32_t lane = threadIdx.x & 31u, warp = threadIdx.x >> 5;
+    uint16_t* d16 = reinterpret_cast<uint16_t*>(dst);
+    uint4* d = reinterpret_cast<uint4*>(dst + 2 * h);
+#pragma unroll 1
+    for (uint32_t q0 = 0; q0 * 31u <= n8; q0 += kWarps * S) {
+        uint4 a[S], b[S];
+#pragma unroll
+        for (int j = 0; j < S; ++j) {
+            const uint32_t blk = (q0 + warp * S + j) * 31u + lane;
+            a[j] = 2 * blk < nvs ? ld_stream(s + 2 * blk) : make_uint4(0u, 0u, 0u, 0u);
+            b[j] = 2 * blk + 1 < nvs ? ld_stream(s + 2 * blk + 1) : make_uint4(0u, 0u, 0u, 0u);
+        }
+#pragma unroll
+        for (int j = 0; j < S; ++j) {
+            const uint32_t blk = (q0 + warp * S + j) * 31u + lane;
+            uint4 o;
+            o.x = pack_bf16x2(a[j].x, a[j].y);
+            o.y = pack_bf16x2(a[j].z, a[j].w);
+            o.z = pack_bf16x2(b[j].x, b[j].y);
+            o.w = pack_bf16x2(b[j].z, b[j].w);
+            uint4 nx;
+            nx.x = __shfl_down_sync(0xFFFFFFFFu, o.x, 1);
+            nx.y = __shfl_down_sync(0xFFFFFFFFu, o.y, 1);
+            nx.z = __shfl_down_sync(0xFFFFFFFFu, o.z, 1);
+            nx.w = __shfl_down_sync(0xFFFFFFFFu, o.w, 1);
+            if (lane < 31u) {
+                if (blk < n8) {
+                    st_stream(d + blk, shift_pick<Q>(o, nx, r));
+                } else if (blk == n8 && tail) {
+                    const uint4 v = shift_pick<Q>(o, nx, r);
+                    const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+                    uint16_t* t = reinterpret_cast<uint16_t*>(d + blk);
+#pragma unroll
+                    for (uint32_t e = 0; e < 7; ++e)
+                        if (e < tail) t[e] = (uint16_t)(w[e >> 1] >> (16 * (e & 1)));
+                }
+            }
+            if (blk == 0) {
+                const uint32_t w[4] = {o.x, o.y, o.z, o.w};
+#pragma unroll
+                for (uint32_t e = 0; e < 7; ++e)
+                    if (e < h) d16[e] = (uint16_t)(w[e >> 1] >> (16 * (e & 1)));
+            }
+        }
+    }
+}
+
+__device__ __noinline__ void cta_cast_shuffled(unsigned char* __restrict__ dst, const unsigned char* __restrict__ src,
+                                               uint32_t len) {
+    constexpr int S = T2I_TUNE_CAST_SHUFFLE_STEPS;
+    static_assert((kThreads / 32) * S * 31 >= kPieceBytes / 32 + 1, "one round covers a piece");
+    const uint32_t nf = len >> 2;
+    const uint32_t h = umin(((16u - (uint32_t)(reinterpret_cast<uintptr_t>(dst) & 15u)) & 15u) >> 1, nf);
+    const uint32_t n8 = (nf - h) >> 3;
+    const uint32_t tail = nf - h - (n8 << 3);
+    const uint32_t nvs = (len + 15) >> 4;
+    const uint4* s = reinterpret_cast<const uint4*>(src);
+    // output halfword e of vector k is halfword h + e of blocks k, k + 1:
+    // a shift of 2h bytes = 4Q + r bytes
+    const uint32_t r = (h & 1u) * 2u;
+    switch (h >> 1) {
+        case 0: emit_cast_shuffled<0, S>(dst, s, h, n8, tail, nvs, r); break;
+        case 1: emit_cast_shuffled<1, S>(dst, s, h, n8, tail, nvs, r); break;
+        case 2: emit_cast_shuffled<2, S>(dst, s, h, n8, tail, nvs, r); break;
+        default: emit_cast_shuffled<3, S>(dst, s, h, n8, tail, nvs, r); break;
+    }
+}
+
 // Largest segment index whose first granule is <= g (segments are non-empty
 // and ordered by start). All threads search the same g: uniform loads.
 __device__ __forceinline__ uint32_t find_segment(const SegDesc* segs, uint32_t n, uint32_t g) {
@@ -639,7 +733,9 @@ __device__ __forceinline__ void run_range(const LaunchParams<BLOB>& p, uint64_t 
         unsigned char* uaddr = reinterpret_cast<unsigned char*>(s.user);
         if (M == Mode::Get || M == Mode::GetCopy) {
             if (M == Mode::Get && (s.nbytes_flags & kCastFlag)) {
-                if (GENERAL)
+                if (GENERAL && T2I_TUNE_CAST_SHUFFLE)
+                    cta_cast_shuffled(uaddr + (off >> 1), paddr, len);
+                else if (GENERAL)
                     cta_cast_staged(uaddr + (off >> 1), paddr, len);
                 else
                     cta_cast_aligned<kV>(uaddr + (off >> 1), paddr, len);

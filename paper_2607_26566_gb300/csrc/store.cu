@@ -353,9 +353,10 @@ t2i_status Store::put(const t2i_put_desc* descs, uint32_t n, t2i_id* ids, cudaSt
                 err_ = "put: item " + std::to_string(i) + ": " + err_;
                 return st;
             }
+            // (without pointer checks the kind of memory is unknown: no prefetch)
             if (!ce && d.nbytes)
-                device_sources = device_sources && !d.src_is_host &&
-                                 (!cfg_.check_pointers || cache.kind == MemKind::Device);
+                device_sources = device_sources && !d.src_is_host && cfg_.check_pointers &&
+                                 cache.kind == MemKind::Device;
         }
         use_ce[i] = ce;
     }
