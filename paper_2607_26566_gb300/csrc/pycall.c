@@ -7,9 +7,12 @@
  * itself on a small request. This module passes the same arguments (plain
  * integers: the store handle, descriptor and id array addresses, counts and
  * the cudaStream_t) to the same C-ABI functions of libt2istore.so with
- * METH_FASTCALL, and keeps the lock for the call (a few microseconds of
- * host work, no blocking wait). Marshalling only: every check, page table
- * step and byte move happens in the library.
+ * METH_FASTCALL, and keeps the interpreter lock for the call: a few
+ * microseconds of host work, unless the call waits for the store's own lock
+ * (another thread is inside the store) or for room in a full launch queue,
+ * during which other Python threads wait too (the ctypes binding releases
+ * the lock instead). Marshalling only: every check, page table step and
+ * byte move happens in the library.
  */
 #define PY_SSIZE_T_CLEAN
 #include <Python.h>
