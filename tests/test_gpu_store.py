@@ -797,3 +797,58 @@ def test_prepared_batches():
         for o in outs:
             o.zero_()
     assert st.stats()["used_pages"] == 0
+
+
+def _cudart():
+    """The CUDA runtime library, to allocate managed memory (torch does not)."""
+    import ctypes
+    import os
+
+    home = os.environ.get("CUDA_HOME") or os.environ.get("CUDA_PATH") or "/usr/local/cuda"
+    for name in ("libcudart.so", "libcudart.so.13", "libcudart.so.12"):
+        for path in (os.path.join(home, "lib64", name), name):
+            try:
+                return ctypes.CDLL(path)
+            except OSError:
+                pass
+    pytest.fail("no CUDA runtime library found to allocate managed memory")
+
+
+def test_puts_the_kernels_do_not_prefetch():
+    """Sources whose bytes the put kernels must not ask L2 for ahead of their
+    wait: managed memory (checked as such), and every source of a store
+    without pointer checks (the kind of memory is unknown). Every get equals
+    the oracle's, and so do the page lists."""
+    import ctypes
+
+    rng = np.random.default_rng(21)
+    P = 64 * 1024
+    datas = [rng.integers(0, 256, int(n), dtype=np.uint8) for n in (1000, 3 * P + 5, 70001, 2 * P, 17)]
+    rt = _cudart()
+    managed = []
+    try:
+        for d in datas:
+            p = ctypes.c_void_p()
+            assert rt.cudaMallocManaged(ctypes.byref(p), ctypes.c_size_t(d.size), 1) == 0
+            ctypes.memmove(p, d.ctypes.data, d.size)  # managed memory is host-accessible
+            managed.append(p.value)
+        for check in (1, 0):
+            st = make_store(64 * P, P, check_pointers=check)
+            ora = OracleStore(64 * P, P)
+            srcs = np.array(managed, np.uint64) if check else [dev_bytes(d, 3 * k) for k, d in enumerate(datas)]
+            s, ids = st.put_batch(put_descs(srcs, nbytes=[d.size for d in datas]))
+            assert s == 0, st.last_error()
+            ost, oids = ora.put_batch([PutItem(d.size, d) for d in datas])
+            assert ost == 0 and list(ids) == oids
+            compare_meta(st, ora)
+            outs = [dev_empty(d.size, k) for k, d in enumerate(datas)]
+            s, _ = st.get_batch(get_descs(oids, outs))
+            assert s == 0, st.last_error()
+            torch.cuda.synchronize()
+            for o, d in zip(outs, datas):
+                assert np.array_equal(host(o), d)
+            st.close()
+    finally:
+        torch.cuda.synchronize()
+        for p in managed:
+            rt.cudaFree(ctypes.c_void_p(p))
