@@ -2040,7 +2040,11 @@ def main():
         # pages, whose gets ended early in the step before, instead of the
         # pages of its last get (LIFO), so steps overlap on the link too
         he.reopen(h2d_mode=1, d2h_mode=1, alloc_policy=1)
-        ms_c2 = dist_ctx.max(time_two_streams(he, e_steps))
+        # three measurements, the median reported: the host link is shared with
+        # the rest of the machine, and one measurement can land in a burst of
+        # someone else's traffic
+        ms_c2_reps = [dist_ctx.max(time_two_streams(he, e_steps)) for _ in range(3)]
+        ms_c2 = statistics.median(ms_c2_reps)
         he.verify()
         gbs = lambda ms: round(job_gbs(he.step_bytes * e_steps, ms, dist_ctx), 2)  # noqa: E731
         e2e = {"value": gbs(ms_c2), "unit": "GB/s",
@@ -2049,6 +2053,7 @@ def main():
                        "for the host copies (h2d_mode = d2h_mode = 1), extent placement (alloc_policy = 1); "
                        "puts on one stream, gets on another",
                "link_gbs": round((he.h2d_bytes + he.d2h_bytes) * e_steps / (ms_c2 * 1e-3) / 1e9, 1),
+               "measurements": [gbs(m) for m in ms_c2_reps],
                "lifo_placement_value": gbs(ms_c2_lifo),
                "kernel_host_copies": {"streams4_value": gbs(ms_e), "one_stream_value": gbs(ms_e1),
                                       "puts_and_gets_on_two_streams_value": gbs(ms_k2)}}

@@ -161,7 +161,7 @@ def test_failed_compaction_still_orders_the_pages_it_wrote():
     torch.cuda.synchronize()
     _late(s1, 30)
     assert st.inject_launch_failure(2) == 0
-    s, moved = st.compact(6000 * P, stream=s1)        # 2,000 one-page moves: two launches
+    s, moved = st.compact(6000 * P, stream=s1)        # 2,000 one-page moves: several launches
     assert s == CUDA and moved == 0
     s, nids = st.put_batch(put_descs(new.data_ptr() + P * np.arange(2000), nbytes=np.full(2000, P)), stream=s2)
     assert s == 0
