@@ -14,7 +14,7 @@
  * binding's cost, and this program's host time per call is the library's
  * own (pointer checks, directory, page dependencies, launch).
  *
- * Usage: handoff_step B [requests streams steps warmup page_bytes pool_gib]
+ * Usage: handoff_step B [requests streams steps warmup page_bytes pool_gib check_pointers]
  * Prints one JSON line: GB/s of the step (algorithmic bytes: 2 x payload for
  * a put, 2 x payload for a copy and 1.5 x payload for the cast in a get) and
  * host microseconds per put and per get call. Inputs are constant bytes per
@@ -56,7 +56,7 @@ static double now_us(void) {
 
 int main(int argc, char** argv) {
     if (argc < 2) {
-        fprintf(stderr, "usage: %s B [requests streams steps warmup page_bytes pool_gib]\n", argv[0]);
+        fprintf(stderr, "usage: %s B [requests streams steps warmup page_bytes pool_gib check_pointers]\n", argv[0]);
         return 1;
     }
     const uint64_t B = strtoull(argv[1], NULL, 10);
@@ -66,6 +66,7 @@ int main(int argc, char** argv) {
     const int warmup = argc > 5 ? atoi(argv[5]) : 3;
     const uint64_t page = argc > 6 ? strtoull(argv[6], NULL, 10) : (2ull << 20);
     const uint64_t pool_bytes = (argc > 7 ? strtoull(argv[7], NULL, 10) : 8ull) << 30;
+    const uint32_t check_pointers = argc > 8 ? (uint32_t)atoi(argv[8]) : 1u;
     if (B < 1 || R < 1 || S < 1 || S > 64 || steps < 1 || warmup < 0) {
         fprintf(stderr, "bad arguments\n");
         return 1;
@@ -84,7 +85,7 @@ int main(int argc, char** argv) {
     memset(&cfg, 0, sizeof cfg);
     cfg.pool_bytes = pool_bytes;
     cfg.page_bytes = page;
-    cfg.check_pointers = 1;
+    cfg.check_pointers = check_pointers;
     t2i_store* h = NULL;
     t2i_status st = t2i_store_create(pool, &cfg, 0, &h);
     if (st != T2I_OK) {
@@ -189,9 +190,9 @@ int main(int argc, char** argv) {
     const double calls = (double)R * steps;
     printf("{\"B\": %llu, \"requests\": %d, \"streams\": %d, \"steps\": %d, \"page_bytes\": %llu, "
            "\"gbs\": %.1f, \"ms_per_step\": %.4f, \"host_us_per_put\": %.3f, \"host_us_per_get\": %.3f, "
-           "\"outputs_ok\": %s}\n",
+           "\"check_pointers\": %u, \"outputs_ok\": %s}\n",
            (unsigned long long)B, R, S, steps, (unsigned long long)page, (put_bytes + get_bytes) * steps / (ms * 1e-3) / 1e9,
-           ms / steps, host_put_us / calls, host_get_us / calls, bad ? "false" : "true");
+           ms / steps, host_put_us / calls, host_get_us / calls, check_pointers, bad ? "false" : "true");
     t2i_store_destroy(h);
     return bad ? 4 : 0;
 }
