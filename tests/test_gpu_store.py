@@ -591,15 +591,20 @@ def test_handoff_spread_over_streams():
     assert st.stats()["used_pages"] == 0
 
 
-@pytest.mark.parametrize("B", [1, 8])
-def test_bench_step_over_streams(B):
+@pytest.mark.parametrize("B,binding", [(1, "cpython"), (8, "cpython"), (1, "ctypes")])
+def test_bench_step_over_streams(B, binding):
     """The benchmark's own multi-stream step (phase joins included), at the
     headline's size and launch configuration (B = 8, 64 requests, 4 streams)
-    and at B = 1: get(put(x)) == x for every output, the oracle's cast for
-    sampled requests."""
+    and at B = 1, through the CPython entry points and through ctypes (the
+    form used where the CPython module was not built): get(put(x)) == x for
+    every output, the oracle's cast for sampled requests."""
     import bench
 
     hw = bench.Handoff(B, W.HANDOFF["requests"], DEV)
+    if binding == "ctypes":
+        hw.fast = None
+    else:
+        assert hw.fast is not None, "the CPython entry points were not built"
     streams = [torch.cuda.current_stream()] + [torch.cuda.Stream() for _ in range(3)]
     for _ in range(3):
         hw.step_streams(streams)
