@@ -126,13 +126,13 @@ def test_adapters_small_vs_oracle():
 
 
 def test_adapters_full_size_vs_oracle():
-    """The full adapter workload (512 sets, 16 GiB pool, 256 KiB pages), its
-    first 3,000 calls on the GPU store: the store evicts exactly the oracle's
-    victims in the oracle's order, reloads as often, and ends with the
-    oracle's free-page stack; every 50th window equals its bank bytes. (All
-    10,000 calls of the trace are replayed on the control core against the
-    oracle in the CPU tests.)"""
-    n = 3000
+    """The full adapter workload (512 sets, 16 GiB pool, 256 KiB pages), all
+    10,000 calls of its trace on the GPU store: the store evicts exactly the
+    oracle's victims in the oracle's order, reloads as often, and ends with
+    the oracle's free-page stack; every 50th window equals its bank bytes.
+    (The CPU tests also compare the control core with the oracle after every
+    call of the same trace.)"""
+    n = W.ADAPTERS["n_calls"]
     ad = bench.Adapters(DEV, n_calls=n)
     for k in range(n):
         s, w = ad.call(k)
@@ -140,7 +140,7 @@ def test_adapters_full_size_vs_oracle():
             m = ad.expected(s, w).numel()
             assert torch.equal(ad.dst[:m], ad.expected(s, w)), k
     oa = _oracle_replay(ad, n)
-    assert len(ad.victims) == len(oa.victims) > 100_000
+    assert len(ad.victims) == len(oa.victims) > 1_000_000
     assert ad.victims == oa.victims
     assert ad.loads == oa.loads
     assert ad.store.ctl.free_pages() == oa.b.free_pages()
