@@ -129,16 +129,15 @@ def test_adapters_full_size_vs_oracle():
     """The full adapter workload (512 sets, 16 GiB pool, 256 KiB pages), all
     10,000 calls of its trace on the GPU store: the store evicts exactly the
     oracle's victims in the oracle's order, reloads as often, and ends with
-    the oracle's free-page stack; every 50th window equals its bank bytes.
+    the oracle's free-page stack; every got window equals its bank bytes.
     (The CPU tests also compare the control core with the oracle after every
     call of the same trace.)"""
     n = W.ADAPTERS["n_calls"]
     ad = bench.Adapters(DEV, n_calls=n)
     for k in range(n):
         s, w = ad.call(k)
-        if k % 50 == 0:
-            m = ad.expected(s, w).numel()
-            assert torch.equal(ad.dst[:m], ad.expected(s, w)), k
+        m = ad.expected(s, w).numel()
+        assert torch.equal(ad.dst[:m], ad.expected(s, w)), k
     oa = _oracle_replay(ad, n)
     assert len(ad.victims) == len(oa.victims) > 1_000_000
     assert ad.victims == oa.victims
