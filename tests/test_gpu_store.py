@@ -401,6 +401,36 @@ def test_error_paths_never_reach_the_gpu():
     assert st.stats()["live_objects"] == 1 and st.stats()["used_pages"] == 1
 
 
+def test_error_paths_through_the_cpython_entry_points():
+    """The same refusals through the CPython entry points (prepared batches'
+    path): bad sources and destinations come back INVALID from the library
+    before any launch, unknown ids NOT_FOUND, and the store is unchanged."""
+    P = 64 * 1024
+    st = make_store(16 * P, P)
+    assert st._fast is not None, "the CPython entry points were not built"
+    stream = int(torch.cuda.current_stream().cuda_stream)
+    x = torch.zeros(1000, dtype=torch.uint8, device=DEV)
+    pp = st.prepare_put(put_descs([x]))
+    s, ids = st.put_prepared(pp)
+    assert s == 0
+    good = int(ids[0])
+    bad_puts = [put_descs([x], nbytes=[10**8]), put_descs([12345], nbytes=[10]),
+                put_descs([st.pool], nbytes=[100])]
+    out = np.zeros(1, np.uint64)
+    for d in bad_puts:
+        assert st._fast.put_batch(st._hi, d.ctypes.data, 1, out.ctypes.data, stream) == 1
+    small = torch.empty(10, dtype=torch.uint8, device=DEV)
+    pg = st.prepare_get(get_descs([0], [small]))
+    assert st.get_prepared(pg, np.array([good], np.uint64)) == 1          # destination too small
+    assert list(pg.descs["id"]) == [good]
+    pg2 = st.prepare_get(get_descs([0], [x]))
+    assert st.get_prepared(pg2, np.array([999], np.uint64)) == 3          # unknown id
+    assert list(pg2.out) == [3]
+    torch.cuda.synchronize()
+    assert st.stats()["live_objects"] == 1 and st.stats()["used_pages"] == 1
+    assert st.stats()["gets"] == 0
+
+
 def test_compaction_moves_bytes_vs_oracle():
     """A fragmented store compacted to a smaller limit and grown back: every
     byte vs the oracle, page lists vs the oracle's paged model."""
