@@ -67,6 +67,8 @@ def parse():
     p.add_argument("--rows-only", action="store_true", help="skip the handoff headline (profiling a row)")
     p.add_argument("--weight-blocks", type=int, default=None,
                    help="restore only the first N blocks into a pool sized for them (profiling small cases)")
+    p.add_argument("--lib", default=None,
+                   help="time this build of libt2istore.so instead of the package's (tuning sweeps)")
     p.add_argument("--compaction-gib", type=int, default=None,
                    help="smaller compaction pool (GiB; the limit is 3/4 of it): profiling small cases")
     return p.parse_args()
@@ -1915,7 +1917,18 @@ def main():
 
     from paper_2607_26566_gb300 import build as b
 
-    b.ensure_built()
+    if args.lib:
+        # a library built with other compile-time launch shapes (tuning
+        # sweeps): every call goes to it through ctypes (the CPython module
+        # is linked against the package's own library)
+        from paper_2607_26566_gb300 import _lib as L
+
+        if L._lib is not None:
+            raise RuntimeError("--lib must be set before the library is loaded")
+        L.LIB_PATH = os.path.abspath(args.lib)
+        L._pycall = None
+    else:
+        b.ensure_built()
     device = torch.device("cuda", dist_ctx.local)
     torch.cuda.set_device(device)
     if args.rows_only:
