@@ -672,7 +672,7 @@ def time_unaligned(device, reps: int = 10, nbytes: int = 1 << 30):
     return out
 
 
-def time_c_driver(steps: int = 50, warmup: int = 3):
+def time_c_driver(device, steps: int = 50, warmup: int = 3):
     """The handoff step driven from C through the C ABI (cdriver/handoff_step.c,
     no Python between calls), 64 requests of 2 MiB pages in an 8 GiB pool:
     B = 1 and 8, on 4 streams and on one. Its host microseconds per call are
@@ -683,8 +683,8 @@ def time_c_driver(steps: int = 50, warmup: int = 3):
     exe = b.build_cdriver()
     out = {"workload": "t2i handoff, 64 requests, 2 MiB pages, 8 GiB pool, driven from C", "runs": []}
     for B, S in ((1, 4), (1, 1), (8, 4), (8, 1)):
-        r = subprocess.run([exe, str(B), "64", str(S), str(steps), str(warmup)], capture_output=True, text=True,
-                           timeout=600)
+        r = subprocess.run([exe, str(B), "64", str(S), str(steps), str(warmup), str(2 << 20), "8", "1",
+                            str(device.index or 0)], capture_output=True, text=True, timeout=600)
         if r.returncode:
             raise RuntimeError(f"C driver B={B} S={S} failed: {r.stderr.strip()[-400:]}")
         d = json.loads(r.stdout.strip().splitlines()[-1])
@@ -1877,7 +1877,7 @@ def run_rows(args, device, peak):
     if "unaligned" in wanted:
         rows["unaligned"] = time_unaligned(device)
     if "cdriver" in wanted:
-        rows["cdriver"] = time_c_driver()
+        rows["cdriver"] = time_c_driver(device)
     if "host" in wanted:
         rows["host"] = time_host_control()
     if "weights" in wanted:

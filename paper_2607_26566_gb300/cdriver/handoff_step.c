@@ -14,7 +14,7 @@
  * binding's cost, and this program's host time per call is the library's
  * own (pointer checks, directory, page dependencies, launch).
  *
- * Usage: handoff_step B [requests streams steps warmup page_bytes pool_gib check_pointers]
+ * Usage: handoff_step B [requests streams steps warmup page_bytes pool_gib check_pointers device]
  * Prints one JSON line: GB/s of the step (algorithmic bytes: 2 x payload for
  * a put, 2 x payload for a copy and 1.5 x payload for the cast in a get) and
  * host microseconds per put and per get call. Inputs are constant bytes per
@@ -56,7 +56,8 @@ static double now_us(void) {
 
 int main(int argc, char** argv) {
     if (argc < 2) {
-        fprintf(stderr, "usage: %s B [requests streams steps warmup page_bytes pool_gib check_pointers]\n", argv[0]);
+        fprintf(stderr, "usage: %s B [requests streams steps warmup page_bytes pool_gib check_pointers device]\n",
+                argv[0]);
         return 1;
     }
     const uint64_t B = strtoull(argv[1], NULL, 10);
@@ -67,7 +68,8 @@ int main(int argc, char** argv) {
     const uint64_t page = argc > 6 ? strtoull(argv[6], NULL, 10) : (2ull << 20);
     const uint64_t pool_bytes = (argc > 7 ? strtoull(argv[7], NULL, 10) : 8ull) << 30;
     const uint32_t check_pointers = argc > 8 ? (uint32_t)atoi(argv[8]) : 1u;
-    if (B < 1 || R < 1 || S < 1 || S > 64 || steps < 1 || warmup < 0) {
+    const int device = argc > 9 ? atoi(argv[9]) : 0;
+    if (B < 1 || R < 1 || S < 1 || S > 64 || steps < 1 || warmup < 0 || device < 0) {
         fprintf(stderr, "bad arguments\n");
         return 1;
     }
@@ -78,7 +80,7 @@ int main(int argc, char** argv) {
     const double put_bytes = 2.0 * payload * R;
     const double get_bytes = (2.0 * (payload - nbytes[cast_obj]) + 1.5 * nbytes[cast_obj]) * R;
 
-    CHECK_CUDA(cudaSetDevice(0));
+    CHECK_CUDA(cudaSetDevice(device));
     void* pool = NULL;
     CHECK_CUDA(cudaMalloc(&pool, pool_bytes));
     t2i_store_config cfg;
@@ -87,7 +89,7 @@ int main(int argc, char** argv) {
     cfg.page_bytes = page;
     cfg.check_pointers = check_pointers;
     t2i_store* h = NULL;
-    t2i_status st = t2i_store_create(pool, &cfg, 0, &h);
+    t2i_status st = t2i_store_create(pool, &cfg, device, &h);
     if (st != T2I_OK) {
         fprintf(stderr, "t2i_store_create failed (%d)\n", (int)st);
         return 3;
